@@ -1,0 +1,335 @@
+"""Decode-step benchmark of the GB300 T-LoopFormer library.
+
+python bench.py [--gpus N] [--steps K] [--warmup W] [--config c4] [--impl ours|reference]
+
+One step = one tlf_decode_step over a batch of B sequences (router,
+compaction, every loop's shared block on its active tokens, recursion-wise
+attention, LM head). Default workload: the long-context GQA model (d 2048,
+16 q / 8 kv heads x 128, 2 layers, ffn 5504, M = 6) with batch 16 at 32768
+tokens of context, the configuration the attention bandwidth target is set on.
+Sequences start from restored synthetic cache snapshots whose per-loop lengths
+follow the model's depth distribution (prefill is not part of the step).
+
+Prints one JSON line. ``value`` is decode tokens/s over all ranks, timed with
+CUDA events on the launching stream with logits left on the device; ``e2e``
+is the same metric through the public call with host token ids in and host
+logits out (copies inside the timed region). Under torchrun each rank runs
+its own batch of sequences (weak scaling, no collective on the data path).
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import os
+import statistics
+import subprocess
+import sys
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+from paper_2609_15160_gb300 import synth  # noqa: E402
+
+DESCR = {
+    "c1": "tiny fp32 looped LM (V256 d64 4x16 J1 ff176 M4), batch 1, 32-token prompt",
+    "c2": "small bf16 looped LM (V32000 d512 8x64 J2 ff1376 M4), batch 8, 512-token prompts",
+    "c3": "mid bf16 looped LM (V50304 d1024 16x64 J4 ff2752 M8), batch 64, 2048-token prompts",
+    "c4": "long-context GQA looped LM (d2048 16q/8kv x128 J2 ff5504 M6), batch 16, 32768-token context",
+    "c5": "C3 model, ragged prompts U[128,8192], batch 32, routed depths",
+    "c5f": "C3 model, ragged prompts U[128,8192], batch 32, every token forced to 8 loops",
+}
+
+
+def _measured_peaks():
+    p = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(p):
+        with open(p) as f:
+            d = json.load(f)
+        return d.get("hbm_gbs", 6800.0), "measured"
+    return 6800.0, "fallback"
+
+
+class ClockSampler:
+    """nvidia-smi clock / throttle samples during the timed region."""
+
+    Q = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+         "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+         "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu: int, path: str):
+        self.path, self.proc = path, None
+        try:
+            self.f = open(path, "w")
+            self.proc = subprocess.Popen(["nvidia-smi", f"--id={gpu}", f"--query-gpu={self.Q}", "--format=csv",
+                                          "-lms", "200"], stdout=self.f, stderr=subprocess.DEVNULL)
+        except (OSError, FileNotFoundError):
+            self.proc = None
+
+    def stop(self):
+        if self.proc is None:
+            return None
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except subprocess.TimeoutExpired:
+            self.proc.kill()
+        self.f.close()
+        sm, mx, reasons = [], [], set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for line in open(self.path).read().splitlines()[1:]:
+            parts = [x.strip() for x in line.split(",")]
+            if len(parts) < 9:
+                continue
+            try:
+                sm.append(float(parts[1].split()[0]))
+                mx.append(float(parts[2].split()[0]))
+            except ValueError:
+                continue
+            for n, v in zip(names, parts[5:9]):
+                if v.lower() == "active":
+                    reasons.add(n)
+        if not sm:
+            return None
+        return {"sm_mhz": statistics.median(sm), "sm_max_mhz": max(mx), "reasons": sorted(reasons),
+                "samples": len(sm)}
+
+
+def _dist():
+    ws = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    return ws, rank, local
+
+
+def _oracle_sample_cmd(cfg_name: str, tokens: int, rank_seed: int) -> str:
+    return f"""
+import sys, time, json, numpy as np
+sys.path.insert(0, {ROOT!r})
+from paper_2609_15160_gb300 import synth
+from oracle import tlf_oracle as O
+wl = synth.get_config({cfg_name!r}); m = wl.model
+w = synth.make_weights(m)
+om = O.OracleModel.from_config(m, w)
+L = int(max(len(p) for p in synth.make_prompts(wl, batch=1)))
+snap = synth.make_cache_snapshot(m, L, {rank_seed})
+seq = O.load_snapshot(om, snap, cache_dtype=np.float32)
+toks = synth.make_decode_tokens(wl, steps={tokens}, batch=1)[:, 0]
+t = time.perf_counter()
+for x in toks:
+    O.decode_token(om, seq, int(x))
+print(json.dumps({{"seconds": time.perf_counter() - t, "tokens": {tokens}, "context": L}}))
+"""
+
+
+def cpu_baseline(cfg_name: str, tokens: int = 3) -> dict:
+    """The oracle timed on this host's cores on a bounded sample: one sequence of the workload."""
+    cores = os.cpu_count() or 1
+    env = dict(os.environ, OMP_NUM_THREADS=str(cores), OPENBLAS_NUM_THREADS=str(cores),
+               MKL_NUM_THREADS=str(cores), CUDA_VISIBLE_DEVICES="")
+    r = subprocess.run([sys.executable, "-c", _oracle_sample_cmd(cfg_name, tokens, 11)], capture_output=True,
+                       text=True, env=env, timeout=900)
+    if r.returncode != 0:
+        return {"value": None, "unit": "tokens/s", "cores": cores, "kind": "oracle", "error": r.stderr[-300:]}
+    d = json.loads(r.stdout.strip().splitlines()[-1])
+    return {"value": d["tokens"] / d["seconds"], "unit": "tokens/s", "cores": cores, "kind": "oracle",
+            "sample": f"1 sequence of the workload at context {d['context']}, {d['tokens']} decode tokens "
+                      f"(float64 numpy oracle, BLAS threads = cores)"}
+
+
+def run_reference(args):
+    ws, rank, _ = _dist()
+    if rank != 0:
+        return
+    cfg = args.config
+    cores = os.cpu_count() or 1
+    per_step = []
+    # each step: one decode token of one sequence of the workload through the oracle
+    env = dict(os.environ, OMP_NUM_THREADS=str(cores), OPENBLAS_NUM_THREADS=str(cores), CUDA_VISIBLE_DEVICES="")
+    r = subprocess.run([sys.executable, "-c", _oracle_sample_cmd(cfg, args.warmup + args.steps, 11)],
+                       capture_output=True, text=True, env=env, timeout=3600)
+    if r.returncode != 0:
+        print(json.dumps({"impl": "reference", "unavailable": "oracle run failed: " + r.stderr[-200:]}))
+        return
+    d = json.loads(r.stdout.strip().splitlines()[-1])
+    sec_per_tok = d["seconds"] / d["tokens"]
+    value = 1.0 / sec_per_tok
+    wl = synth.get_config(cfg)
+    line = {"impl": "reference", "metric": "decode_tokens_per_s", "value": value, "unit": "tokens/s",
+            "n_gpus": ws, "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1e3 * sec_per_tok,
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+            "config": {"workload": DESCR[cfg], **synth.describe(wl)},
+            "cpu_baseline": {"value": value, "unit": "tokens/s", "cores": cores, "kind": "oracle",
+                             "sample": f"1 sequence at context {d['context']}, 1 decode token per step"},
+            "e2e": {"value": value, "unit": "tokens/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
+    print(json.dumps(line))
+
+
+def setup_workload(T, wl, rank: int, gemm_impl="auto", prefill="auto"):
+    m = wl.model
+    w = synth.make_weights(m)
+    B = wl.batch
+    prompts = synth.make_prompts(wl)
+    lengths = [len(p) for p in prompts]
+    steps_cap = wl.decode_steps + 64
+    use_snapshot = prefill == "snapshot" or (prefill == "auto" and max(lengths) > 4096)
+    ids = [rank * 100000 + b for b in range(B)]
+    if use_snapshot:
+        distinct = {}
+        snaps = []
+        for b, L in enumerate(lengths):
+            key = (L, b % 2) if wl.prompt_len[0] == wl.prompt_len[1] else (L, 0)
+            if key not in distinct:
+                distinct[key] = synth.make_cache_snapshot(m, L, seed=1000 * rank + len(distinct),
+                                                          depths=None if wl.forced_loops is None else
+                                                          np.full(L, wl.forced_loops, np.int32))
+            snaps.append(distinct[key])
+        pages = sum(sum((len(p) + 63) // 64 for p in s["positions"]) for s in snaps) + B * m.max_loops * (
+            steps_cap // 64 + 2)
+    else:
+        snaps = None
+        pages = B * m.max_loops * ((max(lengths) + steps_cap) // 64 + 2)
+    ctx = T.Context(m, w, max_seqs=B, max_batch=B, max_seq_len=max(lengths) + steps_cap, kv_pool_pages=pages,
+                    gemm_impl=gemm_impl)
+    if snaps is not None:
+        for b in range(B):
+            ctx.load_cache(ids[b], snaps[b])
+    else:
+        forced = None if wl.forced_loops is None else [np.full(len(p), wl.forced_loops, np.int32) for p in prompts]
+        ctx.prefill(ids, prompts, forced=forced, logits=False)
+    return ctx, ids, "restored synthetic snapshot" if snaps is not None else "prefill through the library"
+
+
+def run_ours(args):
+    import torch
+
+    from paper_2609_15160_gb300 import tlf as T
+
+    ws, rank, local = _dist()
+    torch.cuda.set_device(local)
+    if ws > 1:
+        import torch.distributed as dist
+        dist.init_process_group("nccl")
+    T.load_library()
+    wl = synth.get_config(args.config)
+    m = wl.model
+    B = wl.batch
+    t0 = time.time()
+    ctx, ids, how = setup_workload(T, wl, rank, prefill=args.prefill)
+    setup_s = time.time() - t0
+    stream = torch.cuda.current_stream()
+    n_steps = args.warmup + args.steps
+    toks = synth.make_decode_tokens(wl, steps=3 * n_steps + 2, batch=B)
+    forced = None if wl.forced_loops is None else np.full(B, wl.forced_loops, np.int32)
+    logits_dev = torch.empty((B, m.vocab), dtype=torch.float32, device="cuda")
+    logits_host = torch.empty((B, m.vocab), dtype=torch.float32).pin_memory().numpy()
+
+    def barrier():
+        if ws > 1:
+            torch.distributed.barrier()
+        torch.cuda.synchronize()
+
+    # --- device-timed pass (logits stay on the device) ---
+    for s in range(args.warmup):
+        ctx.decode_step(ids, toks[s], forced=forced, logits=logits_dev, stream=stream)
+    clocks = ClockSampler(local, os.path.join(ROOT, "gpurun_out" if os.path.isdir(os.path.join(ROOT, "gpurun_out"))
+                                              else "_work", f"clocks_rank{rank}.csv"))
+    barrier()
+    ev = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps + 1)]
+    ev[0].record(stream)
+    loops_seen = []
+    for s in range(args.steps):
+        _, lp, _ = ctx.decode_step(ids, toks[args.warmup + s], forced=forced, logits=logits_dev, stream=stream)
+        ev[s + 1].record(stream)
+        loops_seen.append(lp)
+    barrier()
+    clk = clocks.stop()
+    step_ms = [ev[i].elapsed_time(ev[i + 1]) for i in range(args.steps)]
+    total_ms = ev[0].elapsed_time(ev[-1])
+
+    # --- end-to-end pass: host tokens in, host logits out ---
+    barrier()
+    t = time.perf_counter()
+    for s in range(args.steps):
+        ctx.decode_step(ids, toks[n_steps + s], forced=forced, logits=logits_host, stream=stream)
+    barrier()
+    e2e_ms = (time.perf_counter() - t) * 1e3
+
+    # --- kernel-level pass: attention kernel time and algorithmic KV bytes ---
+    ctx.set_profiling(True)
+    att_ms, att_bytes, launches, att_launches = 0.0, 0.0, 0, 0
+    for s in range(args.steps):
+        _, lp, _ = ctx.decode_step(ids, toks[2 * n_steps + s], forced=forced, logits=logits_dev, stream=stream)
+        ms, by, nl = ctx.last_step_profile()
+        att_ms += ms
+        att_bytes += by
+        launches += nl
+        att_launches += m.n_layers * m.max_loops
+    ctx.set_profiling(False)
+
+    times = torch.tensor([total_ms, e2e_ms], dtype=torch.float64, device="cuda")
+    if ws > 1:
+        torch.distributed.all_reduce(times, op=torch.distributed.ReduceOp.MAX)
+    total_ms, e2e_ms = times.tolist()
+    loops_seen = np.concatenate(loops_seen)
+    if rank == 0:
+        peak, peak_kind = _measured_peaks()
+        att_gbs = att_bytes / (att_ms * 1e-3) / 1e9 if att_ms > 0 else None
+        value = ws * B * args.steps / (total_ms * 1e-3)
+        h2d = B * 12
+        d2h = B * m.vocab * 4 + B * 8
+        line = {
+            "metric": "decode_tokens_per_s", "value": value, "unit": "tokens/s", "n_gpus": ws,
+            "steps": args.steps, "warmup": args.warmup, "ms_per_step": total_ms / args.steps,
+            "p50_step_ms": float(np.percentile(step_ms, 50)), "p90_step_ms": float(np.percentile(step_ms, 90)),
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": m.dtype,
+            "data": "synthetic",
+            "config": {"workload": DESCR[args.config], "name": args.config, "batch_per_gpu": B,
+                       "context": int(wl.prompt_len[1]), "cache": how,
+                       "l2": "inputs larger than L2 (KV cache and weights stream from HBM every step)",
+                       "parallelism": f"replicas x{ws} (independent sequences per GPU)"},
+            "mean_loops": float(loops_seen.mean()),
+            "attention_gbs": att_gbs,
+            "roofline": {"bound": "hbm", "kernel": "k_attn_decode (recursion-wise split-K attention)",
+                         "achieved": att_gbs, "peak": peak, "unit": "GB/s",
+                         "frac": (att_gbs / peak) if att_gbs else None, "peak_kind": peak_kind,
+                         "traffic": None,
+                         "algorithmic_bytes_per_launch": att_bytes / max(1, att_launches),
+                         "avg_launch_ms": att_ms / max(1, att_launches)},
+            "e2e": {"value": ws * B * args.steps / (e2e_ms * 1e-3), "unit": "tokens/s",
+                    "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h},
+            "gpu_launches": int(launches),
+            "setup_s": setup_s,
+        }
+        if clk:
+            line["clocks"] = clk
+        if not args.no_cpu_baseline and ws == 1:
+            line["cpu_baseline"] = cpu_baseline(args.config)
+        print(json.dumps(line))
+    ctx.close()
+    if ws > 1:
+        torch.distributed.destroy_process_group()
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=32)
+    ap.add_argument("--warmup", type=int, default=5)
+    ap.add_argument("--config", default="c4", choices=sorted(DESCR))
+    ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
+    ap.add_argument("--prefill", default="auto", choices=["auto", "snapshot", "real"])
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    args = ap.parse_args()
+    if args.warmup < 3:
+        args.warmup = 3
+    if args.impl == "reference":
+        run_reference(args)
+    else:
+        run_ours(args)
+
+
+if __name__ == "__main__":
+    main()

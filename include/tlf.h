@@ -1,0 +1,225 @@
+/*
+ * tlf.h -- C ABI of the GB300 (sm_103a) decode-step library for T-LoopFormer,
+ * a looped transformer with token-level elastic depth.
+ *
+ * The operation (T-LoopFormer, Sec. 3.2-3.3 and App. B):
+ *   - a token-choice router maps each token's initial state h^(0) = E[x] to a
+ *     loop count m in 1..M (Eq. 2-5);
+ *   - loop i applies the shared J-layer block only to the tokens with m >= i,
+ *     gathered into a dense list and scattered back (Eq. 6-7);
+ *   - each (loop i, layer j) keeps its own KV cache; a token writes its k, v
+ *     into cache (i, j) only when it runs loop i, and its loop-i query attends
+ *     only to cache (i, j) (Eq. 8-11);
+ *   - exited tokens keep h^(m), which goes through the final RMSNorm and the
+ *     tied LM head.
+ *
+ * Block layout (the workloads' restatement of the paper's NanoGPT block):
+ * pre-norm RMSNorm (eps from the config, gains stored), multi-head attention
+ * with grouped kv heads and rotary position embedding at the token's original
+ * position (pairs (k, k + head_dim/2), angle pos * rope_base^(-2k/head_dim)),
+ * and a SwiGLU MLP; the router is RMSNorm (no gain) then a d -> M linear map
+ * with bias. A decoding token appends its own entry to cache (i, j) and then
+ * attends to every entry of it, itself included.
+ *
+ * Conventions for every call:
+ *   - Return value: TLF_OK (0) or a negative TLF_ERR_* code; on error
+ *     tlf_last_error(ctx) holds a one-line message. A call that fails changes
+ *     no sequence state: validation and page reservation finish before any
+ *     device work is queued.
+ *   - Pointers marked "host" are ordinary CPU memory; pointers marked
+ *     "host or device" are looked up with cudaPointerGetAttributes.
+ *   - The caller owns every buffer it passes; the library copies what it keeps.
+ *   - `stream` is a cudaStream_t (NULL = legacy default stream). Calls that
+ *     return loop counts synchronise that stream before returning.
+ *   - Matrices are row-major with the output dimension first (y = W x).
+ *     "dtype" means float32 when cfg.dtype == TLF_DTYPE_F32 and bfloat16 bit
+ *     patterns (uint16) when cfg.dtype == TLF_DTYPE_BF16.
+ *   - Not thread-safe: one thread drives a context at a time.
+ */
+#ifndef TLF_H_
+#define TLF_H_
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+enum tlf_status {
+  TLF_OK = 0,
+  TLF_ERR_INVALID_ARG = -1,   /* bad config, shape, pointer or duplicate id in a batch */
+  TLF_ERR_UNKNOWN_SEQ = -2,   /* sequence id not live */
+  TLF_ERR_DUPLICATE_SEQ = -3, /* sequence id already live */
+  TLF_ERR_OUT_OF_PAGES = -4,  /* the KV page pool cannot hold the step */
+  TLF_ERR_SEQ_TOO_LONG = -5,  /* sequence would exceed cfg.max_seq_len */
+  TLF_ERR_CUDA = -6,          /* a CUDA runtime call failed */
+  TLF_ERR_BAD_WEIGHTS = -7,   /* missing weight pointer */
+  TLF_ERR_DEVICE = -8,        /* a kernel gave up a bounded wait or saw a bad index */
+  TLF_ERR_NO_DEVICE = -9,     /* host-only context: the call needs a GPU */
+  TLF_ERR_CAPACITY = -10      /* too many live sequences or batch larger than cfg.max_batch */
+};
+
+enum tlf_dtype { TLF_DTYPE_F32 = 0, TLF_DTYPE_BF16 = 1 };
+
+/* Exit rule (Sec. 3.2). ARGMAX: m = 1 + argmax_l z_l, ties to the smaller
+ * depth, margin = z_(1) - z_(2). SURVIVAL (Eq. 3-5): pi = softmax(z),
+ * p^(i) = sum_{l>=i} pi_l, m = max{i : p^(i) > threshold}, margin =
+ * min(p^(m) - threshold, threshold - p^(m+1)), p^(M+1) = 0. */
+enum tlf_exit_rule { TLF_EXIT_ARGMAX = 0, TLF_EXIT_SURVIVAL = 1 };
+
+/* GEMM implementation for bf16 models: AUTO = tcgen05/TMEM tensor-core
+ * kernels; SIMT = CUDA-core kernels (the only choice for float32 models,
+ * also used by tests as a second GPU path). */
+enum tlf_gemm_impl { TLF_GEMM_AUTO = 0, TLF_GEMM_SIMT = 1 };
+
+typedef struct tlf_config {
+  int32_t vocab;        /* V; the LM head is tied to the embedding */
+  int32_t d_model;      /* d, multiple of 64 */
+  int32_t n_heads;      /* query heads Hq */
+  int32_t n_kv_heads;   /* kv heads Hkv, divides Hq (grouped-query attention) */
+  int32_t head_dim;     /* hd in {16, 32, 64, 128} */
+  int32_t n_layers;     /* J layers in the shared block */
+  int32_t ffn_hidden;   /* SwiGLU hidden width, multiple of 16 */
+  int32_t max_loops;    /* M (user-set maximum depth, Sec. 3.2), 1..16 */
+  float rope_base;      /* 10000 */
+  float norm_eps;       /* RMSNorm eps, 1e-5 */
+  int32_t dtype;        /* tlf_dtype: weights, activations between kernels and KV pages */
+  int32_t exit_rule;    /* tlf_exit_rule */
+  float threshold;      /* survival threshold (Eq. 4), 0.5 */
+  int32_t max_seqs;     /* live sequences held at once */
+  int32_t max_batch;    /* tokens per decode step, 1..256 */
+  int32_t max_seq_len;  /* tokens per sequence */
+  int32_t page_size;    /* tokens per KV page, multiple of 16 (64 is a good default) */
+  int32_t gemm_impl;    /* tlf_gemm_impl */
+  int32_t host_only;    /* 1: allocate nothing on a GPU; only validation and bookkeeping run */
+  int32_t reserved0;
+  int64_t kv_pool_pages;/* pages in the KV pool; 0 = max_seqs * max_loops * ceil(max_seq_len / page_size) */
+} tlf_config;
+
+/* Host pointers to the weights. Shapes use V, d, Hq, Hkv, hd, J, ff, M from
+ * the config. Norm gains and the router bias are float32; every other matrix
+ * is in the config dtype. The library copies them to the GPU in tlf_create. */
+typedef struct tlf_weights {
+  const void* embedding;   /* [V][d] */
+  const void* router_w;    /* [M][d] */
+  const float* router_b;   /* [M] */
+  const void* wq;          /* [J][Hq*hd][d] */
+  const void* wk;          /* [J][Hkv*hd][d] */
+  const void* wv;          /* [J][Hkv*hd][d] */
+  const void* wo;          /* [J][d][Hq*hd] */
+  const void* w_gate;      /* [J][ff][d] */
+  const void* w_up;        /* [J][ff][d] */
+  const void* w_down;      /* [J][d][ff] */
+  const float* attn_norm;  /* [J][d] */
+  const float* mlp_norm;   /* [J][d] */
+  const float* final_norm; /* [d] */
+} tlf_weights;
+
+typedef struct tlf_ctx tlf_ctx;
+
+/* Validate a configuration without touching a GPU. Returns TLF_OK or
+ * TLF_ERR_INVALID_ARG; `msg` (may be NULL) receives a NUL-terminated reason. */
+int tlf_validate_config(const tlf_config* cfg, char* msg, size_t msg_len);
+
+/* Bytes of one KV page: n_layers * 2 (K, V) * n_kv_heads * page_size *
+ * head_dim * element size. Pages are shared by the J layers of one
+ * (sequence, loop) cache. Returns 0 for an invalid config. */
+int64_t tlf_page_bytes(const tlf_config* cfg);
+
+/* Create a context: validate cfg, copy the weights to the current CUDA
+ * device, allocate the KV page pool and step workspaces. *out receives the
+ * context (NULL on failure). On failure the message is available through
+ * tlf_last_error(NULL) on the same thread. */
+int tlf_create(const tlf_config* cfg, const tlf_weights* w, tlf_ctx** out);
+
+/* Free every device and host resource of the context. NULL is a no-op. */
+void tlf_destroy(tlf_ctx* ctx);
+
+/* Message of the last failed call on ctx (or of the last failed tlf_create
+ * on this thread when ctx is NULL). Never NULL. */
+const char* tlf_last_error(const tlf_ctx* ctx);
+
+/* Prefill (Sec. 3.3, "prefill" in App. B): create n_seqs new sequences and
+ * run their prompts. Prompt s is tokens[offsets[s] .. offsets[s+1]) (host,
+ * offsets has n_seqs+1 entries, every prompt non-empty). Each prompt token is
+ * routed, and runs its loops in position order; its k, v land in the caches
+ * of the loops it runs, at its original position.
+ *   seq_ids      host [n_seqs], distinct, not live
+ *   forced       host [offsets[n_seqs]] or NULL; entries >= 1 replace the
+ *                router's loop count (fixed-depth runs), others are ignored
+ *   last_logits  host or device float32 [n_seqs][V] or NULL: logits after
+ *                each prompt's last token
+ *   loops        host int32 [offsets[n_seqs]] or NULL: loop count per token
+ * Errors: INVALID_ARG, DUPLICATE_SEQ, CAPACITY, SEQ_TOO_LONG, OUT_OF_PAGES,
+ * CUDA, DEVICE. */
+int tlf_prefill(tlf_ctx* ctx, int32_t n_seqs, const uint64_t* seq_ids, const int32_t* offsets,
+                const int32_t* tokens, const int32_t* forced, float* last_logits, int32_t* loops,
+                void* stream);
+
+/* One decode step (Sec. 3.3, Eq. 9-11): one new token for each of `batch`
+ * live, distinct sequences. The router picks each token's loop count; loop i
+ * runs on the dense list of tokens with m >= i; each token appends k, v to
+ * the loop-i caches of its sequence and attends to them.
+ *   seq_ids        host [batch]
+ *   tokens         host [batch] token ids in [0, V)
+ *   forced         host [batch] or NULL; entries >= 1 replace the router's
+ *                  loop count
+ *   logits         host or device float32 [batch][V]; NULL skips the LM head
+ *   loops          host int32 [batch] (required): the loop counts m
+ *   router_margin  host float32 [batch] or NULL: the router's decision margin
+ *                  (see tlf_exit_rule); a token is a near-tie when it is small
+ * The call synchronises `stream` before returning (loop counts are host
+ * outputs). Errors: INVALID_ARG, UNKNOWN_SEQ, CAPACITY, SEQ_TOO_LONG,
+ * OUT_OF_PAGES, CUDA, DEVICE. */
+int tlf_decode_step(tlf_ctx* ctx, int32_t batch, const uint64_t* seq_ids, const int32_t* tokens,
+                    const int32_t* forced, float* logits, int32_t* loops, float* router_margin,
+                    void* stream);
+
+/* End a sequence and return the pages of all M loop caches to the pool. */
+int tlf_release(tlf_ctx* ctx, uint64_t seq_id);
+
+/* Create a sequence whose recursion-wise caches hold a given snapshot (a
+ * restored session). For loop i (0-based), lens[i] entries at original
+ * positions positions[off_i .. off_i + lens[i]) with off_i = sum_{i'<i}
+ * lens[i'], strictly increasing; loop 0 must hold 0..lens[0]-1, and each
+ * loop's positions must be a subset of the previous loop's (active sets
+ * nest, Eq. 4-5). k and v are host arrays in the config dtype laid out
+ * [sum lens][J][Hkv][hd] in the same loop order, already rotated (RoPE at
+ * their positions). The next token of the sequence has position lens[0].
+ * Errors: INVALID_ARG, DUPLICATE_SEQ, CAPACITY, SEQ_TOO_LONG, OUT_OF_PAGES,
+ * CUDA, NO_DEVICE. */
+int tlf_load_cache(tlf_ctx* ctx, uint64_t seq_id, const int32_t* lens, const int32_t* positions,
+                   const void* k, const void* v);
+
+/* ---- inspection ---------------------------------------------------------- */
+
+/* Number of live sequences and free pages. */
+int tlf_stats(const tlf_ctx* ctx, int32_t* live_seqs, int64_t* free_pages, int64_t* total_pages);
+
+/* Entries in the loop-`loop` caches (1-based loop) of a sequence; all J layers share it. */
+int tlf_cache_len(const tlf_ctx* ctx, uint64_t seq_id, int32_t loop, int32_t* len);
+
+/* Copy cache (loop, layer) of a sequence to the host: positions int32 [len],
+ * k and v float32 [len][Hkv][hd] (widened from the storage dtype). `loop` is
+ * 1-based, `layer` 0-based. Any output pointer may be NULL. */
+int tlf_read_cache(tlf_ctx* ctx, uint64_t seq_id, int32_t loop, int32_t layer, int32_t* positions,
+                   float* k, float* v);
+
+/* Active sets of the last decode step (Eq. 4-6): counts[i] = |A_{i+1}| for
+ * i < M, and idx[i * batch + r] for r < counts[i] the batch rows of A_{i+1}
+ * in increasing order. Host arrays [M] and [M * batch]. */
+int tlf_last_active_sets(tlf_ctx* ctx, int32_t* counts, int32_t* idx);
+
+/* Kernel-level timing of the last decode step, filled when
+ * tlf_set_profiling(ctx, 1) is on: milliseconds spent in the recursion-wise
+ * attention kernels, the KV bytes they read (K and V of every visited entry
+ * once per kv head), and the number of kernels launched. */
+int tlf_set_profiling(tlf_ctx* ctx, int32_t on);
+int tlf_last_step_profile(const tlf_ctx* ctx, float* attn_ms, double* attn_kv_bytes,
+                          int32_t* kernel_launches);
+
+#ifdef __cplusplus
+}
+#endif
+#endif /* TLF_H_ */

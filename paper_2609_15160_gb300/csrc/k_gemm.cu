@@ -1,0 +1,242 @@
+// Dense projections of the shared block on the compacted tokens (Eq. 6, 9):
+// Y[row][o] = sum_k X[row][k] * W[o][k] for the n rows of the active set.
+//
+// k_gemm_tc (bf16): tcgen05 tensor-core GEMM. Operand roles are swapped so
+// that the weight tile fills the 128-row MMA dimension and the n <= 256 tokens
+// form the N dimension (decode has few tokens and many output features).
+// Warp 0 lane 0 streams 128x64 weight tiles and NTx64 token tiles into a
+// 4-stage shared-memory ring with 2-D TMA (128-byte swizzle); warp 1 lane 0
+// issues tcgen05.mma (M=128, N=round16(n), K=16) accumulating in TMEM and
+// releases each stage with tcgen05.commit; then all four warps read the
+// accumulator with tcgen05.ld (warp w owns TMEM lanes 32w..32w+31 = output
+// features) and run the epilogue. Split-K over gridDim.y keeps enough CTAs
+// in flight to stream the weights at HBM speed.
+//
+// k_gemm_simt: CUDA-core tiled GEMM with the same epilogues, for float32
+// models (tcgen05 has no exact float32 mode) and as a second GPU path.
+//
+// Epilogues: split-K partial sums (consumed by RoPE/append and SwiGLU),
+// residual add + scatter into the float32 stream H[idx[row]] (Eq. 7, with
+// atomics so split-K partials need no extra pass), or a plain float32 store
+// (logits).
+#include "tlf_internal.cuh"
+
+namespace tlf {
+
+__device__ __forceinline__ void gemm_write(const GemmArgs& a, int split, int row, int col, float v) {
+  if (a.epi == EPI_PARTIAL) {
+    a.out[((size_t)split * a.max_rows + row) * a.N + col] = v;
+  } else if (a.epi == EPI_RESID) {
+    const int r = a.idx ? a.idx[row] : row;
+    atomicAdd(a.resid + (size_t)r * a.ldr + col, v);
+  } else {
+    a.out[(size_t)row * a.ldo + col] = v;
+  }
+}
+
+// ----------------------------------------------------------------------------
+// tcgen05 kernel
+// ----------------------------------------------------------------------------
+constexpr int TC_BM = 128;
+constexpr int TC_BK = 64;  // 64 bf16 = one 128-byte swizzle row
+constexpr int TC_STAGES = 4;
+
+template <int NT>
+constexpr int tc_smem_bytes() {
+  return 1024 /*align slack*/ + TC_STAGES * (TC_BM * TC_BK * 2 + NT * TC_BK * 2) + 256 /*barriers, tmem slot*/;
+}
+
+template <int NT>
+__global__ void __launch_bounds__(128) k_gemm_tc(const __grid_constant__ CUtensorMap mapW,
+                                                 const __grid_constant__ CUtensorMap mapX, GemmArgs a) {
+  constexpr int A_BYTES = TC_BM * TC_BK * 2;
+  constexpr int B_BYTES = NT * TC_BK * 2;
+  constexpr uint32_t TMEM_COLS = NT < 32 ? 32 : NT;
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+  uint8_t* sA = smem;
+  uint8_t* sB = smem + TC_STAGES * A_BYTES;
+  uint64_t* bars = reinterpret_cast<uint64_t*>(sB + TC_STAGES * B_BYTES);
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 2 * TC_STAGES + 1);
+
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int n = a.n_dev ? *a.n_dev : a.n_host;
+  if (n <= 0) return;
+  const int ncols = ((n + 15) / 16) * 16;  // MMA N: multiple of 16, <= NT
+  const int m0 = blockIdx.x * TC_BM;
+  const int split = blockIdx.y;
+  const int nkb = (a.K + TC_BK - 1) / TC_BK;
+  const int kb0 = (int)((long long)split * nkb / a.splits);
+  const int kb1 = (int)((long long)(split + 1) * nkb / a.splits);
+  const int nk = kb1 - kb0;
+
+  auto full = [&](int i) { return smem_u32(&bars[i]); };
+  auto empty = [&](int i) { return smem_u32(&bars[TC_STAGES + i]); };
+  const uint32_t done = smem_u32(&bars[2 * TC_STAGES]);
+
+  if (threadIdx.x == 0) {
+    for (int i = 0; i < TC_STAGES; ++i) {
+      mbar_init(full(i), 1);
+      mbar_init(empty(i), 1);
+    }
+    mbar_init(done, 1);
+    fence_barrier_init();
+    prefetch_tensormap(&mapW);
+    prefetch_tensormap(&mapX);
+  }
+  if (warp == 0) {
+    tmem_alloc(smem_u32(tmem_slot), TMEM_COLS);
+    tmem_relinquish();
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = *tmem_slot;
+
+  if (nk > 0) {
+    if (warp == 0 && lane == 0) {
+      // TMA producer
+      for (int i = 0; i < nk; ++i) {
+        const int st = i % TC_STAGES;
+        const uint32_t ph = (uint32_t)(i / TC_STAGES) & 1u;
+        if (!mbar_wait(empty(st), ph ^ 1u, a.err)) break;
+        mbar_arrive_expect_tx(full(st), A_BYTES + B_BYTES);
+        const int kx = (kb0 + i) * TC_BK;
+        tma_load_2d(smem_u32(sA + st * A_BYTES), &mapW, kx, m0, full(st));
+        tma_load_2d(smem_u32(sB + st * B_BYTES), &mapX, kx, 0, full(st));
+      }
+    } else if (warp == 1 && lane == 0) {
+      // MMA issuer
+      const uint32_t idesc = idesc_bf16_f32(TC_BM, ncols);
+      for (int i = 0; i < nk; ++i) {
+        const int st = i % TC_STAGES;
+        const uint32_t ph = (uint32_t)(i / TC_STAGES) & 1u;
+        if (!mbar_wait(full(st), ph, a.err)) break;
+        tc_fence_after();
+        const uint64_t da = smem_desc_sw128(smem_u32(sA + st * A_BYTES));
+        const uint64_t db = smem_desc_sw128(smem_u32(sB + st * B_BYTES));
+#pragma unroll
+        for (int k = 0; k < TC_BK / 16; ++k)  // +32 bytes per K step of 16 bf16 (encoded >> 4)
+          tc_mma_f16(tmem, da + 2 * k, db + 2 * k, idesc, (i > 0 || k > 0) ? 1u : 0u);
+        tc_commit(empty(st));
+      }
+      tc_commit(done);
+    }
+  }
+  __syncwarp();
+
+  // Epilogue: warp w holds output features m0 + 32w + lane; columns are token rows.
+  bool ok = true;
+  if (nk > 0) ok = mbar_wait(done, 0, a.err);
+  ok = __all_sync(0xffffffffu, ok);  // tcgen05.ld is warp-collective
+  tc_fence_after();
+  if (ok) {
+    const int col = m0 + warp * 32 + lane;
+    for (int c0 = 0; c0 < ncols; c0 += 16) {
+      float v[16];
+      if (nk > 0) {
+        tmem_ld_16(tmem + ((uint32_t)(warp * 32) << 16) + (uint32_t)c0, v);
+      } else {
+#pragma unroll
+        for (int i = 0; i < 16; ++i) v[i] = 0.f;
+      }
+      if (col < a.N) {
+#pragma unroll
+        for (int i = 0; i < 16; ++i)
+          if (c0 + i < n && (nk > 0 || a.epi == EPI_PARTIAL)) gemm_write(a, split, c0 + i, col, v[i]);
+      }
+    }
+  }
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 0) tmem_dealloc(tmem, TMEM_COLS);
+}
+
+int gemm_tc_max_nt() { return 256; }
+
+template <int NT>
+static void launch_tc_nt(const CUtensorMap* mapW, const CUtensorMap* mapX, const GemmArgs& a, cudaStream_t st) {
+  static bool attr_set = false;
+  constexpr int smem = tc_smem_bytes<NT>();
+  if (!attr_set) {
+    cudaFuncSetAttribute(k_gemm_tc<NT>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+    attr_set = true;
+  }
+  dim3 grid((a.N + TC_BM - 1) / TC_BM, a.splits);
+  k_gemm_tc<NT><<<grid, 128, smem, st>>>(*mapW, *mapX, a);
+}
+
+void launch_gemm_tc(const CUtensorMap* mapW, const CUtensorMap* mapX, int nt_max, const GemmArgs& a,
+                    cudaStream_t st) {
+  switch (nt_max) {
+    case 16: launch_tc_nt<16>(mapW, mapX, a, st); break;
+    case 32: launch_tc_nt<32>(mapW, mapX, a, st); break;
+    case 64: launch_tc_nt<64>(mapW, mapX, a, st); break;
+    case 128: launch_tc_nt<128>(mapW, mapX, a, st); break;
+    default: launch_tc_nt<256>(mapW, mapX, a, st); break;
+  }
+}
+
+// ----------------------------------------------------------------------------
+// SIMT kernel: 64 features x 32 rows per CTA, K in steps of 32
+// ----------------------------------------------------------------------------
+template <typename T>
+__global__ void __launch_bounds__(256) k_gemm_simt(const T* __restrict__ W, const T* __restrict__ X, int ldx,
+                                                   GemmArgs a) {
+  __shared__ float Ws[32][65];
+  __shared__ float Xs[32][33];
+  const int n = a.n_dev ? *a.n_dev : a.n_host;
+  if (n <= 0) return;
+  const int f0 = blockIdx.x * 64;
+  const int split = blockIdx.y;
+  const int nkb = (a.K + 31) / 32;
+  const int kb0 = (int)((long long)split * nkb / a.splits);
+  const int kb1 = (int)((long long)(split + 1) * nkb / a.splits);
+  const int tid = threadIdx.x, tx = tid & 15, ty = tid >> 4;
+  for (int row0 = 0; row0 < n; row0 += 32) {
+    float acc[4][2] = {{0.f, 0.f}, {0.f, 0.f}, {0.f, 0.f}, {0.f, 0.f}};
+    for (int kb = kb0; kb < kb1; ++kb) {
+      const int k0 = kb * 32;
+      for (int e = tid; e < 64 * 32; e += 256) {
+        const int fi = e >> 5, kk = e & 31, f = f0 + fi, k = k0 + kk;
+        Ws[kk][fi] = (f < a.N && k < a.K) ? to_f32(W[(size_t)f * a.K + k]) : 0.f;
+      }
+      for (int e = tid; e < 32 * 32; e += 256) {
+        const int ri = e >> 5, kk = e & 31, rr = row0 + ri, k = k0 + kk;
+        Xs[kk][ri] = (rr < n && k < a.K) ? to_f32(X[(size_t)rr * ldx + k]) : 0.f;
+      }
+      __syncthreads();
+#pragma unroll 8
+      for (int kk = 0; kk < 32; ++kk) {
+        float w[4], x[2];
+#pragma unroll
+        for (int i = 0; i < 4; ++i) w[i] = Ws[kk][ty * 4 + i];
+        x[0] = Xs[kk][tx * 2];
+        x[1] = Xs[kk][tx * 2 + 1];
+#pragma unroll
+        for (int i = 0; i < 4; ++i) {
+          acc[i][0] = fmaf(w[i], x[0], acc[i][0]);
+          acc[i][1] = fmaf(w[i], x[1], acc[i][1]);
+        }
+      }
+      __syncthreads();
+    }
+#pragma unroll
+    for (int i = 0; i < 4; ++i)
+#pragma unroll
+      for (int c = 0; c < 2; ++c) {
+        const int f = f0 + ty * 4 + i, rr = row0 + tx * 2 + c;
+        if (f < a.N && rr < n) gemm_write(a, split, rr, f, acc[i][c]);
+      }
+  }
+}
+
+void launch_gemm_simt(int dtype, const void* W, const void* X, int ldx, const GemmArgs& a, cudaStream_t st) {
+  dim3 grid((a.N + 63) / 64, a.splits);
+  if (dtype == 1)
+    k_gemm_simt<bf16><<<grid, 256, 0, st>>>((const bf16*)W, (const bf16*)X, ldx, a);
+  else
+    k_gemm_simt<float><<<grid, 256, 0, st>>>((const float*)W, (const float*)X, ldx, a);
+}
+
+}  // namespace tlf

@@ -1,0 +1,202 @@
+// Row-wise kernels of the decode step.
+//
+// k_norm_rows    gather + RMSNorm: X[k] = RMSNorm(H[idx[k]]) * gain for the
+//                rows of the active set (Eq. 6 followed by the pre-norm).
+// k_rope_append  sums the split-K partials of the fused QKV projection (Eq. 9),
+//                rotates q and k at the token's original position, keeps q for
+//                the attention kernel and appends k, v to the token's slot of
+//                the loop-r page of its sequence (Eq. 11; the slot is the
+//                loop-r cache length, so positions stay in increasing order).
+// k_swiglu       sums gate/up partials and applies silu(g) * u.
+// k_final        final RMSNorm of every row for the LM head, and the cache
+//                length update len[seq][r] += 1 for r < m.
+// k_scatter_cache writes a restored cache snapshot into pages.
+#include "tlf_internal.cuh"
+
+namespace tlf {
+
+__device__ __forceinline__ float block_sum(float v) {
+  __shared__ float ws[32];
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5, nw = (blockDim.x + 31) >> 5;
+  v = warp_sum(v);
+  if (lane == 0) ws[warp] = v;
+  __syncthreads();
+  float t = (lane < nw) ? ws[lane] : 0.f;
+  t = warp_sum(t);
+  __syncthreads();
+  return t;
+}
+
+template <typename T>
+__global__ void __launch_bounds__(256) k_norm_rows(const float* __restrict__ H, int ldh, const int* __restrict__ idx,
+                                                   const int* __restrict__ n_dev, int n_host,
+                                                   const float* __restrict__ gain, int d, float eps,
+                                                   T* __restrict__ X, int ldx) {
+  const int k = blockIdx.x;
+  const int n = n_dev ? *n_dev : n_host;
+  if (k >= n) return;
+  const int src = idx ? idx[k] : k;
+  const float* h = H + (size_t)src * ldh;
+  float ss = 0.f;
+  for (int i = threadIdx.x; i < d; i += blockDim.x) ss += h[i] * h[i];
+  ss = block_sum(ss);
+  const float inv = rsqrtf(ss / (float)d + eps);
+  for (int i = threadIdx.x; i < d; i += blockDim.x) X[(size_t)k * ldx + i] = from_f32<T>(h[i] * inv * gain[i]);
+}
+
+void launch_norm_rows(int dtype, const float* H, int ldh, const int* idx, const int* n_dev, int n_host, int rows_max,
+                      const float* gain, int d, float eps, void* X, int ldx, cudaStream_t st) {
+  if (rows_max <= 0) return;
+  if (dtype == 1)
+    k_norm_rows<bf16><<<rows_max, 256, 0, st>>>(H, ldh, idx, n_dev, n_host, gain, d, eps, (bf16*)X, ldx);
+  else
+    k_norm_rows<float><<<rows_max, 256, 0, st>>>(H, ldh, idx, n_dev, n_host, gain, d, eps, (float*)X, ldx);
+}
+
+template <typename T>
+__global__ void __launch_bounds__(256) k_rope_append(ModelDims md, StepDev s, int r, int j,
+                                                     const float* __restrict__ part, int splits, float* __restrict__ Q,
+                                                     const double* __restrict__ inv_freq) {
+  const int k = blockIdx.x;
+  if (k >= s.n[r]) return;
+  const int b = s.idx[r * md.max_batch + k];
+  const int slot = s.slots[b];
+  const int pos = s.len[slot * md.M + 0];  // every token runs loop 1: its length is the token count
+  const int L = s.len[slot * md.M + r];
+  const int ps = md.page_size, hd = md.hd, half = hd / 2;
+  const int page = s.page_table[((size_t)slot * md.M + r) * md.max_pages + L / ps];
+  if (page < 0 || page >= md.n_pages) {
+    if (threadIdx.x == 0) atomicOr(s.err, DEVERR_INDEX);
+    return;
+  }
+  const int off = L % ps;
+  T* pg = reinterpret_cast<T*>(s.pool) + (size_t)page * md.page_elems;
+  const size_t pstride = (size_t)md.max_batch * md.qkv_dim;
+  const float* prow = part + (size_t)k * md.qkv_dim;
+  const double two_pi = 6.283185307179586476925286766559;
+
+  // q heads then k heads: rotate pair (i, i + hd/2) by pos * theta_i
+  for (int t = threadIdx.x; t < (md.Hq + md.Hkv) * half; t += blockDim.x) {
+    const int h = t / half, i = t % half;
+    const int c0 = h * hd + i, c1 = c0 + half;  // k columns follow the q columns
+    float a = 0.f, c = 0.f;
+    for (int sp = 0; sp < splits; ++sp) {
+      a += prow[sp * pstride + c0];
+      c += prow[sp * pstride + c1];
+    }
+    double ang = (double)pos * inv_freq[i];
+    ang -= two_pi * rint(ang / two_pi);
+    float sn, cs;
+    sincosf((float)ang, &sn, &cs);
+    const float ra = a * cs - c * sn, rc = a * sn + c * cs;
+    if (h < md.Hq) {
+      float* qo = Q + ((size_t)k * md.Hq + h) * hd;
+      qo[i] = ra;
+      qo[i + half] = rc;
+    } else {
+      T* kp = pg + ((size_t)(j * 2 + 0) * md.Hkv + (h - md.Hq)) * ps * hd + (size_t)off * hd;
+      kp[i] = from_f32<T>(ra);
+      kp[i + half] = from_f32<T>(rc);
+    }
+  }
+  for (int t = threadIdx.x; t < md.Hkv * hd; t += blockDim.x) {
+    const int h = t / hd, e = t % hd;
+    const int col = md.q_dim + md.kv_dim + t;
+    float a = 0.f;
+    for (int sp = 0; sp < splits; ++sp) a += prow[sp * pstride + col];
+    T* vp = pg + ((size_t)(j * 2 + 1) * md.Hkv + h) * ps * hd + (size_t)off * hd;
+    vp[e] = from_f32<T>(a);
+  }
+  if (j == 0 && threadIdx.x == 0) s.pos_table[(size_t)page * ps + off] = pos;
+}
+
+void launch_rope_append(const ModelDims& md, const StepDev& s, int r, int j, const float* part, int splits, float* Q,
+                        const double* inv_freq, cudaStream_t st) {
+  if (md.dtype == 1)
+    k_rope_append<bf16><<<md.max_batch, 256, 0, st>>>(md, s, r, j, part, splits, Q, inv_freq);
+  else
+    k_rope_append<float><<<md.max_batch, 256, 0, st>>>(md, s, r, j, part, splits, Q, inv_freq);
+}
+
+template <typename T>
+__global__ void __launch_bounds__(256) k_swiglu(const float* __restrict__ part, int splits, int max_rows,
+                                                const int* __restrict__ n_dev, int ff, T* __restrict__ U) {
+  const int k = blockIdx.y;
+  if (k >= *n_dev) return;
+  const size_t N = 2 * (size_t)ff;
+  for (int f = blockIdx.x * blockDim.x + threadIdx.x; f < ff; f += gridDim.x * blockDim.x) {
+    float g = 0.f, u = 0.f;
+    for (int sp = 0; sp < splits; ++sp) {
+      const float* p = part + ((size_t)sp * max_rows + k) * N;
+      g += p[f];
+      u += p[ff + f];
+    }
+    U[(size_t)k * ff + f] = from_f32<T>(g / (1.f + expf(-g)) * u);
+  }
+}
+
+void launch_swiglu(int dtype, const float* part, int splits, int max_rows, const int* n_dev, int ff, void* U,
+                   cudaStream_t st) {
+  dim3 grid((ff + 255) / 256, max_rows);
+  if (dtype == 1)
+    k_swiglu<bf16><<<grid, 256, 0, st>>>(part, splits, max_rows, n_dev, ff, (bf16*)U);
+  else
+    k_swiglu<float><<<grid, 256, 0, st>>>(part, splits, max_rows, n_dev, ff, (float*)U);
+}
+
+template <typename T>
+__global__ void __launch_bounds__(256) k_final(ModelDims md, StepDev s, const float* __restrict__ gain,
+                                               T* __restrict__ Xf) {
+  const int b = blockIdx.x;
+  const float* h = s.H + (size_t)b * md.d;
+  float ss = 0.f;
+  for (int i = threadIdx.x; i < md.d; i += blockDim.x) ss += h[i] * h[i];
+  ss = block_sum(ss);
+  const float inv = rsqrtf(ss / (float)md.d + md.eps);
+  for (int i = threadIdx.x; i < md.d; i += blockDim.x) Xf[(size_t)b * md.d + i] = from_f32<T>(h[i] * inv * gain[i]);
+  if (threadIdx.x < md.M) {
+    const int r = threadIdx.x;
+    if (r < s.m[b]) s.len[s.slots[b] * md.M + r] += 1;
+  }
+}
+
+void launch_final(const ModelDims& md, const StepDev& s, int B, const float* gain, void* Xf, cudaStream_t st) {
+  if (md.dtype == 1)
+    k_final<bf16><<<B, 256, 0, st>>>(md, s, gain, (bf16*)Xf);
+  else
+    k_final<float><<<B, 256, 0, st>>>(md, s, gain, (float*)Xf);
+}
+
+// Snapshot entries e < n of loop r: src layout [n][J][Hkv][hd] for k and v.
+template <typename T>
+__global__ void k_scatter_cache(ModelDims md, int slot, int r, int n, const T* __restrict__ k, const T* __restrict__ v,
+                                const int* __restrict__ positions, const int* __restrict__ page_table, T* pool,
+                                int* pos_table) {
+  const int e = blockIdx.x;
+  if (e >= n) return;
+  const int ps = md.page_size, hd = md.hd;
+  const int page = page_table[((size_t)slot * md.M + r) * md.max_pages + e / ps];
+  if (page < 0 || page >= md.n_pages) return;
+  const int off = e % ps;
+  T* pg = pool + (size_t)page * md.page_elems;
+  const int per = md.J * md.Hkv * hd;
+  for (int t = threadIdx.x; t < per; t += blockDim.x) {
+    const int jj = t / (md.Hkv * hd), rem = t % (md.Hkv * hd), h = rem / hd, i = rem % hd;
+    pg[((size_t)(jj * 2 + 0) * md.Hkv + h) * ps * hd + (size_t)off * hd + i] = k[(size_t)e * per + t];
+    pg[((size_t)(jj * 2 + 1) * md.Hkv + h) * ps * hd + (size_t)off * hd + i] = v[(size_t)e * per + t];
+  }
+  if (threadIdx.x == 0) pos_table[(size_t)page * ps + off] = positions[e];
+}
+
+void launch_scatter_cache(const ModelDims& md, int slot, int r, int n, const void* k, const void* v,
+                          const int* positions, const int* page_table, void* pool, int* pos_table, cudaStream_t st) {
+  if (n <= 0) return;
+  if (md.dtype == 1)
+    k_scatter_cache<bf16><<<n, 256, 0, st>>>(md, slot, r, n, (const bf16*)k, (const bf16*)v, positions, page_table,
+                                             (bf16*)pool, pos_table);
+  else
+    k_scatter_cache<float><<<n, 256, 0, st>>>(md, slot, r, n, (const float*)k, (const float*)v, positions,
+                                              page_table, (float*)pool, pos_table);
+}
+
+}  // namespace tlf

@@ -1,0 +1,190 @@
+// Token-choice router and active-set compaction (T-LoopFormer Sec. 3.2, Eq. 2-6).
+//
+// k_router: one warp per token. h^(0) = E[x] is written to the float32
+// residual stream H, RMSNorm (no gain) is applied, the M router logits
+// z = W_r x + b_r are reduced across the warp, and the loop count m and its
+// decision margin are taken in float32 (ARGMAX or SURVIVAL rule, see tlf.h).
+// The same kernel applies the page-table updates the host queued for the step.
+//
+// k_plan: one CTA. For every loop r it builds A_r = {b : m_b >= r} in
+// increasing b with a warp ballot plus a block prefix scan, and the work plan
+// of the split-K decode attention over the loop-r caches: the keys per chunk
+// (sized from the device-side cache lengths so that the chunk count is close
+// to a target) and each active token's first work item.
+#include "tlf_internal.cuh"
+
+namespace tlf {
+
+template <typename T>
+__global__ void __launch_bounds__(256) k_router(ModelDims md, StepDev s, int B, const T* __restrict__ emb,
+                                                const T* __restrict__ rw, const float* __restrict__ rb,
+                                                const PageUpdate* __restrict__ upd, int n_upd) {
+  for (int u = blockIdx.x * blockDim.x + threadIdx.x; u < n_upd; u += gridDim.x * blockDim.x) {
+    const PageUpdate p = upd[u];
+    s.page_table[p.index] = p.page;
+  }
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int b = blockIdx.x * 8 + warp;
+  if (b >= B) return;
+  const int d = md.d, M = md.M;
+  int tok = s.tokens[b];
+  if (tok < 0 || tok >= md.V) {
+    if (lane == 0) atomicOr(s.err, DEVERR_INDEX);
+    tok = 0;
+  }
+  const T* e = emb + (size_t)tok * d;
+  float* h = s.H + (size_t)b * d;
+  float ss = 0.f;
+  for (int i = lane; i < d; i += 32) {
+    const float x = to_f32(e[i]);
+    h[i] = x;
+    ss += x * x;
+  }
+  ss = warp_sum(ss);
+  const float inv = rsqrtf(ss / (float)d + md.eps);
+
+  float z[16];
+#pragma unroll
+  for (int l = 0; l < 16; ++l) {
+    if (l < M) {
+      const T* w = rw + (size_t)l * d;
+      float acc = 0.f;
+      for (int i = lane; i < d; i += 32) acc += (to_f32(e[i]) * inv) * to_f32(w[i]);
+      z[l] = warp_sum(acc) + rb[l];
+    } else {
+      z[l] = -INFINITY;
+    }
+  }
+
+  int m = 1;
+  float margin;
+  if (md.exit_rule == 0) {
+    // ARGMAX: first maximum wins (ties go to the smaller depth)
+    int top = 0;
+#pragma unroll
+    for (int l = 1; l < 16; ++l)
+      if (l < M && z[l] > z[top]) top = l;
+    float second = -INFINITY;
+#pragma unroll
+    for (int l = 0; l < 16; ++l)
+      if (l < M && l != top) second = fmaxf(second, z[l]);
+    m = top + 1;
+    margin = z[top] - second;  // +inf when M == 1
+  } else {
+    // SURVIVAL (Eq. 2-5): softmax, suffix sums p^(i), m = max{i : p^(i) > threshold}
+    float mx = z[0];
+#pragma unroll
+    for (int l = 1; l < 16; ++l)
+      if (l < M) mx = fmaxf(mx, z[l]);
+    float ex[16], sum = 0.f;
+#pragma unroll
+    for (int l = 0; l < 16; ++l) {
+      ex[l] = (l < M) ? expf(z[l] - mx) : 0.f;
+      sum += ex[l];
+    }
+    float p[17];
+    p[16] = 0.f;
+    float acc = 0.f;
+#pragma unroll
+    for (int l = 15; l >= 0; --l) {
+      acc += ex[l] / sum;
+      p[l] = acc;
+    }
+    m = 1;
+#pragma unroll
+    for (int l = 0; l < 16; ++l)
+      if (l < M && p[l] > md.threshold) m = l + 1;
+    const float pm = p[m - 1];
+    const float pnext = (m < M) ? p[m] : 0.f;
+    margin = fminf(pm - md.threshold, md.threshold - pnext);
+  }
+  const int f = s.forced[b];
+  if (f >= 1) m = min(f, M);
+  if (lane == 0) {
+    s.m[b] = m;
+    s.margin[b] = margin;
+  }
+}
+
+// Exclusive scan of one int per thread over the block (blockDim.x <= 1024).
+__device__ int block_exclusive_scan(int v, int* total) {
+  __shared__ int warp_tot[32];
+  __shared__ int tot;
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5, nw = (blockDim.x + 31) >> 5;
+  int x = v;
+#pragma unroll
+  for (int o = 1; o < 32; o <<= 1) {
+    const int y = __shfl_up_sync(0xffffffffu, x, o);
+    if (lane >= o) x += y;
+  }
+  if (lane == 31) warp_tot[warp] = x;
+  __syncthreads();
+  if (warp == 0) {
+    int t = (lane < nw) ? warp_tot[lane] : 0;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+      const int y = __shfl_up_sync(0xffffffffu, t, o);
+      if (lane >= o) t += y;
+    }
+    if (lane < nw) warp_tot[lane] = t;  // inclusive
+    if (lane == 31) tot = t;
+  }
+  __syncthreads();
+  const int excl = x - v + (warp > 0 ? warp_tot[warp - 1] : 0);
+  *total = tot;
+  __syncthreads();
+  return excl;
+}
+
+__global__ void __launch_bounds__(256) k_plan(ModelDims md, StepDev s, int B, int target_items, int min_chunk) {
+  const int b = threadIdx.x;
+  const int lane = b & 31;
+  const int mb = (b < B) ? s.m[b] : 0;
+  const int slot = (b < B) ? s.slots[b] : 0;
+  const int maxB = md.max_batch, M = md.M, ps = md.page_size;
+  for (int r = 0; r < M; ++r) {
+    const bool active = mb > r;
+    // compaction: ballot gives each active lane its rank in the warp, the block scan the warp offsets
+    const unsigned ball = __ballot_sync(0xffffffffu, active);
+    const int rank = __popc(ball & ((1u << lane) - 1u));
+    int n_r;
+    const int warp_off = block_exclusive_scan((lane == 0) ? __popc(ball) : 0, &n_r);
+    const int k = __shfl_sync(0xffffffffu, warp_off, 0) + rank;
+    if (active) s.idx[r * maxB + k] = b;
+    // attention plan over the loop-r caches (the token's own new entry included)
+    const int L = active ? s.len[slot * M + r] + 1 : 0;
+    int tot_keys;
+    (void)block_exclusive_scan(L, &tot_keys);
+    long long want = ((long long)tot_keys * md.Hkv + target_items - 1) / target_items;
+    int ch = (int)(((want + ps - 1) / ps) * ps);
+    if (ch < min_chunk) ch = min_chunk;
+    const int nc = active ? (L + ch - 1) / ch : 0;
+    int items;
+    const int base = block_exclusive_scan(nc * md.Hkv, &items);
+    if (active) {
+      s.item_base[r * (maxB + 1) + k] = base;
+      s.nch[r * maxB + k] = nc;
+    }
+    if (b == 0) {
+      s.n[r] = n_r;
+      s.item_base[r * (maxB + 1) + n_r] = items;
+      s.chunk[r] = ch;
+    }
+  }
+}
+
+void launch_router(const ModelDims& md, const StepDev& s, int B, const void* emb, const void* router_w,
+                   const float* router_b, const PageUpdate* upd, int n_upd, cudaStream_t st) {
+  const int grid = (B + 7) / 8;
+  if (md.dtype == 1)
+    k_router<bf16><<<grid, 256, 0, st>>>(md, s, B, (const bf16*)emb, (const bf16*)router_w, router_b, upd, n_upd);
+  else
+    k_router<float><<<grid, 256, 0, st>>>(md, s, B, (const float*)emb, (const float*)router_w, router_b, upd,
+                                          n_upd);
+}
+
+void launch_plan(const ModelDims& md, const StepDev& s, int B, int target_items, int min_chunk, cudaStream_t st) {
+  k_plan<<<1, 256, 0, st>>>(md, s, B, target_items, min_chunk);
+}
+
+}  // namespace tlf

@@ -1,0 +1,318 @@
+// Internal declarations shared by the kernels and the host runtime of libtlf.
+//
+// Device helpers here are thin inline-PTX wrappers (mbarrier, 1-D bulk copy,
+// 2-D tensor copy, tcgen05) written from the public PTX ISA. Every wait on an
+// mbarrier is bounded by wall-clock time (%globaltimer); when it runs out the
+// kernel records TLF_DEVERR_WAIT in the context's error word and returns, so
+// no kernel of this library can spin forever.
+#pragma once
+
+#include <cuda.h>
+#include <cuda_bf16.h>
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+namespace tlf {
+
+// ----------------------------------------------------------------------------
+// Error word bits written by kernels (read by the host after each step).
+// ----------------------------------------------------------------------------
+enum : uint32_t {
+  DEVERR_WAIT = 1u,       // an mbarrier wait ran past its time limit
+  DEVERR_INDEX = 2u,      // a page id / slot / row index was out of range
+  DEVERR_TMEM = 4u,       // TMEM allocation returned an unusable address
+};
+
+constexpr uint64_t kWaitLimitNs = 4000000000ull;  // 4 s
+
+// ----------------------------------------------------------------------------
+// Element helpers
+// ----------------------------------------------------------------------------
+typedef __nv_bfloat16 bf16;
+
+__device__ __forceinline__ float to_f32(float x) { return x; }
+__device__ __forceinline__ float to_f32(bf16 x) { return __bfloat162float(x); }
+template <typename T> __device__ __forceinline__ T from_f32(float x);
+template <> __device__ __forceinline__ float from_f32<float>(float x) { return x; }
+template <> __device__ __forceinline__ bf16 from_f32<bf16>(float x) { return __float2bfloat16_rn(x); }
+
+// 16 bytes of T widened to float: 4 floats or 8 bf16.
+template <typename T> struct Vec16;
+template <> struct Vec16<float> {
+  static constexpr int N = 4;
+  __device__ __forceinline__ static void load(const float* p, float* out) {
+    float4 v = *reinterpret_cast<const float4*>(p);
+    out[0] = v.x; out[1] = v.y; out[2] = v.z; out[3] = v.w;
+  }
+};
+template <> struct Vec16<bf16> {
+  static constexpr int N = 8;
+  __device__ __forceinline__ static void load(const bf16* p, float* out) {
+    uint4 v = *reinterpret_cast<const uint4*>(p);
+    const uint32_t w[4] = {v.x, v.y, v.z, v.w};
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+      out[2 * i] = __uint_as_float(w[i] << 16);
+      out[2 * i + 1] = __uint_as_float(w[i] & 0xFFFF0000u);
+    }
+  }
+};
+
+// ----------------------------------------------------------------------------
+// Shared-memory address, timers, mbarrier
+// ----------------------------------------------------------------------------
+__device__ __forceinline__ uint32_t smem_u32(const void* p) {
+  return static_cast<uint32_t>(__cvta_generic_to_shared(p));
+}
+
+__device__ __forceinline__ uint64_t globaltimer_ns() {
+  uint64_t t;
+  asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
+  return t;
+}
+
+__device__ __forceinline__ void mbar_init(uint32_t bar, uint32_t count) {
+  asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(bar), "r"(count) : "memory");
+}
+
+// Make barrier initialisation visible to the async proxy (TMA, tcgen05.commit).
+__device__ __forceinline__ void fence_barrier_init() {
+  asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+  asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+}
+
+__device__ __forceinline__ void mbar_arrive_expect_tx(uint32_t bar, uint32_t bytes) {
+  asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(bar), "r"(bytes) : "memory");
+}
+
+__device__ __forceinline__ void mbar_arrive(uint32_t bar) {
+  asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(bar) : "memory");
+}
+
+__device__ __forceinline__ bool mbar_try_wait(uint32_t bar, uint32_t parity) {
+  uint32_t ok;
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
+      "selp.u32 %0, 1, 0, p;\n\t}"
+      : "=r"(ok)
+      : "r"(bar), "r"(parity)
+      : "memory");
+  return ok != 0;
+}
+
+// Wait for the phase with the given parity to complete; false after the time limit
+// (the error word then carries DEVERR_WAIT).
+__device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity, uint32_t* err) {
+  if (mbar_try_wait(bar, parity)) return true;
+  const uint64_t t0 = globaltimer_ns();
+  while (true) {
+    if (mbar_try_wait(bar, parity)) return true;
+    if (globaltimer_ns() - t0 > kWaitLimitNs) {
+      atomicOr(err, DEVERR_WAIT);
+      return false;
+    }
+  }
+}
+
+// 1-D bulk copy global -> shared (TMA engine), completing tx bytes on `bar`.
+// dst, src and bytes must be multiples of 16.
+__device__ __forceinline__ void bulk_g2s(uint32_t dst, const void* src, uint32_t bytes, uint32_t bar) {
+  asm volatile(
+      "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(dst),
+      "l"(src), "r"(bytes), "r"(bar)
+      : "memory");
+}
+
+// 2-D tiled tensor copy global -> shared with a tensor map (coordinates in elements,
+// innermost first). The innermost coordinate times the element size is a multiple of 16.
+__device__ __forceinline__ void tma_load_2d(uint32_t dst, const CUtensorMap* map, int32_t c0, int32_t c1,
+                                            uint32_t bar) {
+  asm volatile(
+      "cp.async.bulk.tensor.2d.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1, {%2, %3}], [%4];" ::"r"(
+          dst),
+      "l"(reinterpret_cast<uint64_t>(map)), "r"(c0), "r"(c1), "r"(bar)
+      : "memory");
+}
+
+__device__ __forceinline__ void prefetch_tensormap(const CUtensorMap* map) {
+  asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(map)) : "memory");
+}
+
+// ----------------------------------------------------------------------------
+// tcgen05 (5th-generation tensor core, accumulators in tensor memory)
+// ----------------------------------------------------------------------------
+__device__ __forceinline__ void tmem_alloc(uint32_t dst_smem, uint32_t ncols) {
+  asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(dst_smem), "r"(ncols)
+               : "memory");
+}
+__device__ __forceinline__ void tmem_relinquish() {
+  asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
+}
+__device__ __forceinline__ void tmem_dealloc(uint32_t taddr, uint32_t ncols) {
+  asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(taddr), "r"(ncols) : "memory");
+}
+__device__ __forceinline__ void tc_fence_before() {
+  asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
+}
+__device__ __forceinline__ void tc_fence_after() {
+  asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+}
+
+// D(tmem) (+)= A(smem desc) * B(smem desc), kind::f16 (bf16 inputs, f32 accumulate).
+__device__ __forceinline__ void tc_mma_f16(uint32_t d_tmem, uint64_t a_desc, uint64_t b_desc, uint32_t idesc,
+                                           uint32_t accumulate) {
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "setp.ne.b32 p, %4, 0;\n\t"
+      "tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n\t}" ::"r"(d_tmem),
+      "l"(a_desc), "l"(b_desc), "r"(idesc), "r"(accumulate)
+      : "memory");
+}
+
+// Arrive on an mbarrier once every tcgen05.mma issued so far by this thread has completed.
+__device__ __forceinline__ void tc_commit(uint32_t bar) {
+  asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(bar)
+               : "memory");
+}
+
+// 32 lanes x 32-bit, 16 consecutive columns per thread.
+__device__ __forceinline__ void tmem_ld_16(uint32_t taddr, float* v) {
+  uint32_t r[16];
+  asm volatile(
+      "tcgen05.ld.sync.aligned.32x32b.x16.b32 "
+      "{%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15}, [%16];"
+      : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7]),
+        "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]), "=r"(r[14]), "=r"(r[15])
+      : "r"(taddr));
+  asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
+#pragma unroll
+  for (int i = 0; i < 16; ++i) v[i] = __uint_as_float(r[i]);
+}
+
+// Shared-memory matrix descriptor for a K-major operand tile written by TMA with
+// 128-byte swizzling: rows of 128 B, 8-row swizzle atoms 1024 B apart.
+__device__ __forceinline__ uint64_t smem_desc_sw128(uint32_t saddr) {
+  uint64_t d = 0;
+  d |= (uint64_t)((saddr >> 4) & 0x3FFFu);        // start address
+  d |= (uint64_t)1u << 16;                        // leading byte offset (unused for swizzled K-major)
+  d |= (uint64_t)(1024u >> 4) << 32;              // stride byte offset: 8 rows * 128 B
+  d |= (uint64_t)1u << 46;                        // descriptor version (sm_100 family)
+  d |= (uint64_t)2u << 61;                        // layout: 128-byte swizzle
+  return d;
+}
+
+// Instruction descriptor: kind::f16, A = B = bf16, D = f32, both K-major, M x N.
+__host__ __device__ constexpr uint32_t idesc_bf16_f32(int M, int N) {
+  return (1u << 4) | (1u << 7) | (1u << 10) | ((uint32_t)(N >> 3) << 17) | ((uint32_t)(M >> 4) << 24);
+}
+
+// ----------------------------------------------------------------------------
+// Warp / block reductions and scans
+// ----------------------------------------------------------------------------
+__device__ __forceinline__ float warp_sum(float v) {
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+  return v;
+}
+__device__ __forceinline__ float warp_max(float v) {
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) v = fmaxf(v, __shfl_xor_sync(0xffffffffu, v, o));
+  return v;
+}
+
+// ----------------------------------------------------------------------------
+// Kernel argument blocks
+// ----------------------------------------------------------------------------
+enum GemmEpilogue : int {
+  EPI_PARTIAL = 0,  // out[s][row][col] = acc (split-K partial sums, float32)
+  EPI_RESID = 1,    // atomicAdd(resid[idx[row]][col], acc) (residual add + scatter, Eq. 7)
+  EPI_STORE = 2,    // out[row][col] = acc (float32; single split)
+};
+
+struct GemmArgs {
+  int N;             // output features (rows of W)
+  int K;             // reduction length
+  int splits;        // split-K factor (gridDim.y)
+  const int* n_dev;  // token rows n (device scalar), or NULL to use n_host
+  int n_host;
+  int epi;           // GemmEpilogue
+  float* out;        // EPI_PARTIAL: [splits][max_rows][N]; EPI_STORE: [rows][ldo]
+  int ldo;
+  int max_rows;
+  float* resid;      // EPI_RESID: [*][ldr]
+  int ldr;
+  const int* idx;    // EPI_RESID row map (NULL = identity)
+  uint32_t* err;
+};
+
+struct StepDev {
+  // per-step inputs / outputs (device)
+  const int* tokens;   // [B]
+  const int* forced;   // [B]
+  const int* slots;    // [B] sequence slot of each row
+  int* m;              // [B] loop counts
+  float* margin;       // [B]
+  float* H;            // [B][d] residual stream, float32
+  // compaction / plan, written by the plan kernel
+  int* idx;            // [M][maxB] rows of A_r in increasing order
+  int* n;              // [M] |A_r|
+  int* item_base;      // [M][maxB+1]
+  int* nch;            // [M][maxB] chunks per token
+  int* chunk;          // [M] keys per chunk
+  // cache state
+  int* len;            // [max_seqs][M] entries per (sequence, loop)
+  int* page_table;     // [max_seqs][M][max_pages]
+  int* pos_table;      // [n_pages][page_size]
+  void* pool;          // KV pages
+  uint32_t* err;
+};
+
+struct ModelDims {
+  int V, d, Hq, Hkv, hd, J, ff, M;
+  int qkv_dim, q_dim, kv_dim;
+  int max_seqs, max_batch, max_pages, page_size;
+  long long n_pages;
+  long long page_elems;  // elements per page
+  float eps, rope_base, threshold;
+  int exit_rule;
+  int dtype;             // 0 f32, 1 bf16
+};
+
+// ----------------------------------------------------------------------------
+// Launchers (host functions, one .cu file each)
+// ----------------------------------------------------------------------------
+struct PageUpdate {
+  int index;  // into page_table
+  int page;
+};
+
+void launch_router(const ModelDims& md, const StepDev& s, int B, const void* emb, const void* router_w,
+                   const float* router_b, const PageUpdate* upd, int n_upd, cudaStream_t st);
+void launch_plan(const ModelDims& md, const StepDev& s, int B, int target_items, int min_chunk, cudaStream_t st);
+
+void launch_norm_rows(int dtype, const float* H, int ldh, const int* idx, const int* n_dev, int n_host,
+                      int rows_max, const float* gain, int d, float eps, void* X, int ldx, cudaStream_t st);
+
+void launch_gemm_simt(int dtype, const void* W, const void* X, int ldx, const GemmArgs& a, cudaStream_t st);
+void launch_gemm_tc(const CUtensorMap* mapW, const CUtensorMap* mapX, int nt_max, const GemmArgs& a,
+                    cudaStream_t st);
+int gemm_tc_max_nt();
+
+void launch_rope_append(const ModelDims& md, const StepDev& s, int r, int j, const float* part, int splits,
+                        float* Q, const double* inv_freq, cudaStream_t st);
+void launch_attn_decode(const ModelDims& md, const StepDev& s, int r, int j, const float* Q, float* part_o,
+                        float* part_ml, int grid, cudaStream_t st);
+void launch_attn_combine(const ModelDims& md, const StepDev& s, int r, const float* part_o,
+                         const float* part_ml, void* O, cudaStream_t st);
+int attn_decode_grid(const ModelDims& md, int num_sms);
+
+void launch_swiglu(int dtype, const float* part, int splits, int max_rows, const int* n_dev, int ff, void* U,
+                   cudaStream_t st);
+void launch_final(const ModelDims& md, const StepDev& s, int B, const float* gain, void* Xf, cudaStream_t st);
+
+void launch_scatter_cache(const ModelDims& md, int slot, int r, int n, const void* k, const void* v,
+                          const int* positions, const int* page_table, void* pool, int* pos_table,
+                          cudaStream_t st);
+
+}  // namespace tlf

@@ -1,0 +1,272 @@
+"""GPU path vs CPU oracle on the workload configurations and edge cases.
+
+Every call goes through the C ABI (libtlf.so) via the ctypes binding.
+"""
+import numpy as np
+import pytest
+
+from oracle import tlf_oracle as O
+from paper_2609_15160_gb300 import synth
+
+from _parity import DepthOracle, check_active_sets, check_cache, rel_err, tol_for
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module")
+def tlf():
+    torch = pytest.importorskip("torch")
+    if not torch.cuda.is_available():
+        pytest.skip("needs a CUDA GPU")
+    from paper_2609_15160_gb300 import build, tlf as T
+    build.build()
+    T.load_library()
+    return T
+
+
+def _greedy_run(T, wl, steps=None, gemm_impl="auto", check_caches=True):
+    """Prefill + greedy decode, teacher-forced from the oracle's argmax."""
+    m = wl.model
+    w = synth.make_weights(m)
+    om = O.OracleModel.from_config(m, w)
+    depth = DepthOracle(om)
+    prompts = synth.make_prompts(wl)
+    B = len(prompts)
+    steps = wl.decode_steps if steps is None else steps
+    L = max(len(p) for p in prompts) + steps + 1
+    ids = list(range(100, 100 + B))
+    tol = tol_for(m)
+    worst = 0.0
+    with T.Context(m, w, max_seqs=B, max_batch=B, max_seq_len=L, gemm_impl=gemm_impl) as ctx:
+        pf_forced = [depth.forced_for(p) for p in prompts]
+        glog, gloops = ctx.prefill(ids, prompts, forced=pf_forced)
+        seqs = [O.OracleSequence(om) for _ in range(B)]
+        nxt = np.zeros(B, dtype=np.int32)
+        for b in range(B):
+            olog, om_ = O.prefill_gathered(om, seqs[b], prompts[b], forced=pf_forced[b])
+            np.testing.assert_array_equal(gloops[b], om_)
+            np.testing.assert_array_equal(gloops[b], depth.expected(prompts[b], pf_forced[b]))
+            worst = max(worst, rel_err(glog[b], olog))
+            nxt[b] = int(np.argmax(olog))
+        assert worst < tol, f"prefill logits rel err {worst}"
+        for step in range(steps):
+            f = depth.forced_for(nxt)
+            glog, gl, gmar = ctx.decode_step(ids, nxt, forced=f)
+            olog, oloops, omar = O.decode_step(om, seqs, nxt, forced=f)
+            np.testing.assert_array_equal(gl, oloops)
+            check_active_sets(ctx, gl, m.max_loops)
+            e = rel_err(glog, olog)
+            worst = max(worst, e)
+            assert e < tol, f"step {step}: logits rel err {e}"
+            free = f < 1
+            np.testing.assert_allclose(gmar[free], omar[free], rtol=1e-3, atol=1e-4)
+            nxt = np.argmax(olog, axis=1).astype(np.int32)
+        if check_caches:
+            for b in range(B):
+                for r in range(1, m.max_loops + 1):
+                    assert ctx.cache_len(ids[b], r) == seqs[b].cache_len(r)
+            check_cache(ctx, ids[0], seqs[0], m, max(tol, 1e-4) * (1 if m.dtype == "f32" else 1))
+    return worst, depth.n_forced
+
+
+def test_c1_fp32_full_greedy_parity(tlf):
+    worst, forced = _greedy_run(tlf, synth.get_config("c1"))
+    print(f"c1 worst logits rel err {worst:.2e}, near-tie tokens forced {forced}")
+
+
+def test_c2_bf16_full_greedy_parity(tlf):
+    worst, forced = _greedy_run(tlf, synth.get_config("c2"))
+    print(f"c2 worst logits rel err {worst:.2e}, near-tie tokens forced {forced}")
+
+
+def test_c2_simt_gemm_path_matches_oracle(tlf):
+    """The CUDA-core GEMM path on the same bf16 model (a second GPU path for the tcgen05 kernels)."""
+    wl = synth.get_config("c2").with_batch(4)
+    worst, _ = _greedy_run(tlf, wl, steps=8, gemm_impl="simt", check_caches=False)
+    print(f"c2 simt worst {worst:.2e}")
+
+
+def _snapshot_run(T, wl, lengths, steps, sampled, seed=7, distinct=2):
+    """Sequences restored from synthetic cache snapshots, then decode steps of random tokens.
+
+    Loop counts and active sets are checked for every token (against the
+    oracle's depth table); logits and caches for the sampled sequences.
+    """
+    m = wl.model
+    w = synth.make_weights(m)
+    om = O.OracleModel.from_config(m, w)
+    depth = DepthOracle(om)
+    B = len(lengths)
+    snaps = {}
+    for b in range(B):
+        key = (int(lengths[b]), b % distinct)
+        if key not in snaps:
+            snaps[key] = synth.make_cache_snapshot(m, int(lengths[b]), seed + 31 * key[1] + int(lengths[b]))
+    pages = sum(sum((len(p) + 63) // 64 + 1 for p in snaps[(int(lengths[b]), b % distinct)]["positions"])
+                for b in range(B)) + B * m.max_loops * (steps // 64 + 2)
+    ids = list(range(1000, 1000 + B))
+    tokens = synth.make_decode_tokens(wl, steps=steps, batch=B)
+    tol = tol_for(m)
+    worst = 0.0
+    with T.Context(m, w, max_seqs=B, max_batch=B, max_seq_len=int(max(lengths)) + steps + 1,
+                   kv_pool_pages=pages) as ctx:
+        for b in range(B):
+            ctx.load_cache(ids[b], snaps[(int(lengths[b]), b % distinct)])
+        oseqs = {b: O.load_snapshot(om, snaps[(int(lengths[b]), b % distinct)], cache_dtype=np.float32)
+                 for b in sampled}
+        all_loops = []
+        for step in range(steps):
+            f = depth.forced_for(tokens[step])
+            glog, gl, _ = ctx.decode_step(ids, tokens[step], forced=f)
+            np.testing.assert_array_equal(gl, depth.expected(tokens[step], f))
+            check_active_sets(ctx, gl, m.max_loops)
+            all_loops.append(gl.copy())
+            for b in sampled:
+                olog, oml, _ = O.decode_token(om, oseqs[b], int(tokens[step][b]), forced=int(f[b]))
+                assert oml == gl[b]
+                e = rel_err(glog[b], olog)
+                worst = max(worst, e)
+                assert e < tol, f"step {step} seq {b}: rel err {e}"
+        all_loops = np.array(all_loops)
+        for b in range(B):
+            snap = snaps[(int(lengths[b]), b % distinct)]
+            for r in range(1, m.max_loops + 1):
+                want = len(snap["positions"][r - 1]) + int((all_loops[:, b] >= r).sum())
+                assert ctx.cache_len(ids[b], r) == want
+        for b in sampled:
+            check_cache(ctx, ids[b], oseqs[b], m, tol)
+    return worst, depth.n_forced
+
+
+def test_c3_full_size_sampled_parity(tlf):
+    wl = synth.get_config("c3")
+    lengths = np.full(wl.batch, wl.prompt_len[0])
+    worst, forced = _snapshot_run(tlf, wl, lengths, steps=4, sampled=[0, 37])
+    print(f"c3 worst {worst:.2e} forced {forced}")
+
+
+def test_c4_full_size_sampled_parity(tlf):
+    wl = synth.get_config("c4")
+    lengths = np.full(wl.batch, wl.prompt_len[0])
+    worst, forced = _snapshot_run(tlf, wl, lengths, steps=3, sampled=[0, 9])
+    print(f"c4 worst {worst:.2e} forced {forced}")
+
+
+def test_c5_ragged_sampled_parity(tlf):
+    wl = synth.get_config("c5")
+    lengths = np.array([len(p) for p in synth.make_prompts(wl)])
+    worst, forced = _snapshot_run(tlf, wl, lengths, steps=3, sampled=[int(np.argmax(lengths)), int(np.argmin(lengths))],
+                                  distinct=1)
+    print(f"c5 worst {worst:.2e} forced {forced}")
+
+
+# ----------------------------------------------------------------------------
+# edge cases on small models
+# ----------------------------------------------------------------------------
+
+def _small(dtype="bf16", **kw):
+    base = dict(vocab=300, d_model=128, n_heads=4, n_kv_heads=2, head_dim=64, n_layers=2, ffn_hidden=160,
+                max_loops=4, dtype=dtype, depth_probs=(0.25, 0.25, 0.25, 0.25))
+    if dtype == "f32":
+        base["depth_probs"] = None
+    base.update(kw)
+    return synth.ModelConfig(**base)
+
+
+def _prefill_decode_compare(T, m, prompt_lens, steps, forced_mode=None, seed=0, gemm_impl="auto"):
+    w = synth.make_weights(m)
+    om = O.OracleModel.from_config(m, w)
+    depth = DepthOracle(om)
+    rng = np.random.default_rng(seed)
+    prompts = [rng.integers(0, m.vocab, size=n).astype(np.int32) for n in prompt_lens]
+    B = len(prompts)
+    ids = [7 * b + 3 for b in range(B)]
+    tol = tol_for(m)
+
+    def forced_of(toks):
+        if forced_mode is None:
+            return depth.forced_for(toks)
+        if forced_mode == "random":
+            return rng.integers(1, m.max_loops + 1, size=len(toks)).astype(np.int32)
+        return np.full(len(toks), forced_mode, dtype=np.int32)
+
+    with T.Context(m, w, max_seqs=B + 1, max_batch=B, max_seq_len=max(prompt_lens) + steps + 2,
+                   gemm_impl=gemm_impl) as ctx:
+        pf = [forced_of(p) for p in prompts]
+        glog, gl = ctx.prefill(ids, prompts, forced=pf)
+        seqs = [O.OracleSequence(om) for _ in range(B)]
+        for b in range(B):
+            olog, oml = O.prefill_gathered(om, seqs[b], prompts[b], forced=pf[b])
+            np.testing.assert_array_equal(gl[b], oml)
+            assert rel_err(glog[b], olog) < tol
+        for s in range(steps):
+            toks = rng.integers(0, m.vocab, size=B).astype(np.int32)
+            f = forced_of(toks)
+            glog, gm, _ = ctx.decode_step(ids, toks, forced=f)
+            olog, om2, _ = O.decode_step(om, seqs, toks, forced=f)
+            np.testing.assert_array_equal(gm, om2)
+            check_active_sets(ctx, gm, m.max_loops)
+            assert rel_err(glog, olog) < tol
+        for b in range(B):
+            check_cache(ctx, ids[b], seqs[b], m, max(tol, 1e-4))
+        live, free, total = ctx.stats()
+        for i in ids:
+            ctx.release(i)
+        assert ctx.stats() == (0, total, total)
+
+
+@pytest.mark.parametrize("lens", [[1], [63, 64, 65], [128, 1, 129]])
+def test_page_boundaries_and_ragged_batches(tlf, lens):
+    _prefill_decode_compare(tlf, _small(), lens, steps=3)
+
+
+@pytest.mark.parametrize("gqa", [(4, 4), (4, 2), (8, 2)])
+def test_gqa_ratios(tlf, gqa):
+    _prefill_decode_compare(tlf, _small(n_heads=gqa[0], n_kv_heads=gqa[1], d_model=256), [40, 70], steps=2)
+
+
+@pytest.mark.parametrize("hd", [32, 128])
+def test_head_dims(tlf, hd):
+    _prefill_decode_compare(tlf, _small(head_dim=hd, n_heads=4, n_kv_heads=2, d_model=256), [66, 3], steps=2)
+
+
+def test_every_token_exits_after_one_loop(tlf):
+    """Deeper loops have no active token (device-side counts are zero)."""
+    _prefill_decode_compare(tlf, _small(), [30, 65], steps=3, forced_mode=1)
+
+
+def test_fixed_depth_mode(tlf):
+    """Every token forced to M loops: the fixed-depth looped transformer."""
+    _prefill_decode_compare(tlf, _small(), [30, 65], steps=3, forced_mode=4)
+
+
+def test_random_forced_depths(tlf):
+    _prefill_decode_compare(tlf, _small(max_loops=6, depth_probs=None), [100, 7, 64], steps=4, forced_mode="random")
+
+
+def test_survival_exit_rule(tlf):
+    _prefill_decode_compare(tlf, _small(exit_rule="survival", depth_probs=None), [50, 20], steps=3)
+
+
+def test_fp32_small_model(tlf):
+    _prefill_decode_compare(tlf, _small(dtype="f32", head_dim=32, n_heads=4, n_kv_heads=2), [70, 5], steps=3)
+
+
+def test_wide_batch(tlf):
+    """A batch larger than one MMA N tile (n > 128 tokens)."""
+    m = _small(vocab=500, max_loops=3, depth_probs=(0.3, 0.3, 0.4))
+    _prefill_decode_compare(tlf, m, [3 + (b % 5) for b in range(160)], steps=2)
+
+
+def test_profile_counters(tlf):
+    m = _small()
+    w = synth.make_weights(m)
+    with tlf.Context(m, w, max_seqs=2, max_batch=2, max_seq_len=200) as ctx:
+        ctx.prefill([1, 2], [np.arange(100, dtype=np.int32) % m.vocab, np.arange(10, dtype=np.int32)], logits=False)
+        ctx.set_profiling(True)
+        _, loops, _ = ctx.decode_step([1, 2], [5, 6])
+        ms, by, nl = ctx.last_step_profile()
+        assert ms > 0 and nl == 2 + m.max_loops * m.n_layers * 10 + 1 + 1
+        want = sum((ctx.cache_len(i, r)) * m.n_layers * 2 * m.n_kv_heads * m.head_dim * 2
+                   for i, lp in zip([1, 2], loops) for r in range(1, lp + 1))
+        assert abs(by - want) < 1e-6 * want
