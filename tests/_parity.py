@@ -53,13 +53,33 @@ def check_active_sets(ctx, loops, M):
         np.testing.assert_array_equal(sets[r], want)
 
 
-def check_cache(ctx, seq_id, oseq, model, tol):
+def cache_tol(model):
+    """Tolerance of a stored K/V entry row (max abs diff / row max).
+
+    An entry of loop i is an intermediate result: it carries the error that
+    bf16 activations accumulate over up to M x J layer applications (the same
+    error the logits carry) plus one bf16 storage rounding (<= 2^-9 of the
+    entry), and a K/V row is normalised by the max of far fewer values than a
+    logits row. So the logits bound is widened by half for bf16 models.
+    """
+    return 1e-4 if model.dtype == "f32" else 3e-2
+
+
+def check_cache(ctx, seq_id, oseq, model, tol=None):
     """GPU cache of one sequence against the oracle's: positions exact, K/V within tol."""
+    tol = cache_tol(model) if tol is None else tol
     for i in range(model.max_loops):
         for j in range(model.n_layers):
             gp, gk, gv = ctx.read_cache(seq_id, i + 1, j)
             op, ok, ov = oseq.caches[i][j].view()
             np.testing.assert_array_equal(gp, op)
-            if len(op):
-                assert rel_err(gk.reshape(len(op), -1), ok.reshape(len(op), -1)) < tol
-                assert rel_err(gv.reshape(len(op), -1), ov.reshape(len(op), -1)) < tol
+            for name, g, o in (("k", gk, ok), ("v", gv, ov)):
+                if not len(op):
+                    continue
+                g2, o2 = g.reshape(len(op), -1).astype(np.float64), o.reshape(len(op), -1).astype(np.float64)
+                row = np.max(np.abs(g2 - o2), axis=1) / np.max(np.abs(o2), axis=1)
+                bad = int(np.argmax(row))
+                assert row[bad] < tol, (f"cache {name} loop {i + 1} layer {j}: entry {bad}/{len(op)} "
+                                        f"(pos {op[bad]}) rel err {row[bad]:.3e}; rows over tol: "
+                                        f"{np.nonzero(row >= tol)[0][:10].tolist()} gpu {g2[bad, :4]} "
+                                        f"oracle {o2[bad, :4]}")

@@ -65,7 +65,7 @@ def _greedy_run(T, wl, steps=None, gemm_impl="auto", check_caches=True):
             for b in range(B):
                 for r in range(1, m.max_loops + 1):
                     assert ctx.cache_len(ids[b], r) == seqs[b].cache_len(r)
-            check_cache(ctx, ids[0], seqs[0], m, max(tol, 1e-4) * (1 if m.dtype == "f32" else 1))
+            check_cache(ctx, ids[0], seqs[0], m)
     return worst, depth.n_forced
 
 
@@ -134,7 +134,7 @@ def _snapshot_run(T, wl, lengths, steps, sampled, seed=7, distinct=2):
                 want = len(snap["positions"][r - 1]) + int((all_loops[:, b] >= r).sum())
                 assert ctx.cache_len(ids[b], r) == want
         for b in sampled:
-            check_cache(ctx, ids[b], oseqs[b], m, tol)
+            check_cache(ctx, ids[b], oseqs[b], m)
     return worst, depth.n_forced
 
 
@@ -208,7 +208,7 @@ def _prefill_decode_compare(T, m, prompt_lens, steps, forced_mode=None, seed=0, 
             check_active_sets(ctx, gm, m.max_loops)
             assert rel_err(glog, olog) < tol
         for b in range(B):
-            check_cache(ctx, ids[b], seqs[b], m, max(tol, 1e-4))
+            check_cache(ctx, ids[b], seqs[b], m)
         live, free, total = ctx.stats()
         for i in ids:
             ctx.release(i)
