@@ -313,8 +313,64 @@ def run_ours(args):
         torch.distributed.destroy_process_group()
 
 
+def run_attn_op(args):
+    """The recursion-wise attention kernels alone (tlf_attn_decode) on C4 shapes: GB/s of K/V streamed."""
+    import torch
+
+    from paper_2609_15160_gb300 import tlf as T
+
+    T.load_library()
+    n, L = args.batch, args.context
+    hq, hkv, hd, J = 16, 8, 128, 2
+    rng = np.random.default_rng(5)
+    need = (L + 63) // 64
+    n_pages = n * need + 1
+    # pool of bf16 bit patterns of multiples of 1/64 in [-2, 2), built without a float32 copy
+    table = (np.arange(-128, 128, dtype=np.float32) / 64.0).view(np.uint32) >> 16
+    pool = torch.empty((n_pages, J, 2, hkv, 64, hd), dtype=torch.int16, device="cuda")
+    for p0 in range(0, n_pages, 256):
+        p1 = min(n_pages, p0 + 256)
+        codes = rng.integers(0, 256, size=(p1 - p0, J, 2, hkv, 64, hd), dtype=np.int16)
+        pool[p0:p1] = torch.from_numpy(table[codes].astype(np.uint16).view(np.int16))
+    pt = torch.from_numpy(rng.permutation(n_pages)[: n * need].reshape(n, need).astype(np.int32)).cuda()
+    lens = torch.full((n,), L, dtype=torch.int32, device="cuda")
+    q = torch.randn((n, hq, hd), dtype=torch.float32, device="cuda")
+    out = torch.empty((n, hq * hd), dtype=torch.int16, device="cuda")
+    err = torch.zeros(4, dtype=torch.int32, device="cuda")
+    a = T.attn_args(n, hq, hkv, hd, J, 1, "bf16", need, n_pages, q, pool, pt, lens, out, err)
+    nbytes = T.tlf_attn_decode_scratch_bytes(a)
+    scratch = torch.empty(nbytes, dtype=torch.uint8, device="cuda")
+    stream = torch.cuda.current_stream()
+    for _ in range(args.warmup):
+        T.tlf_attn_decode(a, scratch, nbytes, stream)
+    torch.cuda.synchronize()
+    ev = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps + 1)]
+    ev[0].record(stream)
+    for s in range(args.steps):
+        T.tlf_attn_decode(a, scratch, nbytes, stream)
+        ev[s + 1].record(stream)
+    torch.cuda.synchronize()
+    assert int(err[0].item()) == 0, "device error word set"
+    ms = [ev[i].elapsed_time(ev[i + 1]) for i in range(args.steps)]
+    kv_bytes = n * L * hkv * hd * 2 * 2
+    io_bytes = n * hq * hd * (4 + 2)
+    peak, kind = _measured_peaks()
+    med = float(np.median(ms))
+    gbs = (kv_bytes + io_bytes) / (med * 1e-3) / 1e9
+    print(json.dumps({"metric": "attention_op_gbs", "value": gbs, "unit": "GB/s", "steps": args.steps,
+                      "warmup": args.warmup, "ms_per_call_p50": med, "higher_is_better": True,
+                      "config": {"op": "tlf_attn_decode", "rows": n, "keys_per_row": L, "hq": hq, "hkv": hkv,
+                                 "head_dim": hd, "dtype": "bf16", "l2": "K/V larger than L2"},
+                      "roofline": {"bound": "hbm", "achieved": gbs, "peak": peak, "unit": "GB/s",
+                                   "frac": gbs / peak, "peak_kind": kind,
+                                   "algorithmic_bytes_per_call": kv_bytes + io_bytes}}))
+
+
 def main():
     ap = argparse.ArgumentParser()
+    ap.add_argument("--op", default=None, choices=["attn"], help="time one kernel-level operation alone")
+    ap.add_argument("--batch", type=int, default=16)
+    ap.add_argument("--context", type=int, default=32768)
     ap.add_argument("--gpus", type=int, default=1)
     ap.add_argument("--steps", type=int, default=32)
     ap.add_argument("--warmup", type=int, default=5)
@@ -325,7 +381,9 @@ def main():
     args = ap.parse_args()
     if args.warmup < 3:
         args.warmup = 3
-    if args.impl == "reference":
+    if args.op == "attn":
+        run_attn_op(args)
+    elif args.impl == "reference":
         run_reference(args)
     else:
         run_ours(args)

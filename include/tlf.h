@@ -192,6 +192,47 @@ int tlf_release(tlf_ctx* ctx, uint64_t seq_id);
 int tlf_load_cache(tlf_ctx* ctx, uint64_t seq_id, const int32_t* lens, const int32_t* positions,
                    const void* k, const void* v);
 
+/* ---- kernel-level operation: recursion-wise decode attention ------------- */
+
+/* One query per row against that row's KV cache (Eq. 10 on a cache that
+ * holds only valid entries, so no mask is needed): for row b and query head
+ * h, out[b][h] = softmax(q[b][h] . K_b^T / sqrt(hd)) V_b over the first
+ * lens[b] entries of the cache addressed by page_table[b], kv head
+ * h / (n_heads / n_kv_heads). The same split-K kernels serve tlf_decode_step.
+ * All pointers are device pointers. Page layout, in the dtype:
+ * [n_pages][n_layers][2 (K, V)][n_kv_heads][page_size][head_dim]; entry e of
+ * row b sits in page page_table[b * max_pages + e / page_size] at offset
+ * e % page_size. */
+typedef struct tlf_attn_args {
+  int32_t n;            /* rows (queries), 1..256 */
+  int32_t n_heads;      /* Hq */
+  int32_t n_kv_heads;   /* Hkv, divides Hq */
+  int32_t head_dim;     /* hd (same choices as tlf_config) */
+  int32_t n_layers;     /* layers stored per page */
+  int32_t layer;        /* layer whose K/V are read, 0..n_layers-1 */
+  int32_t page_size;    /* 64 */
+  int32_t dtype;        /* tlf_dtype of the pool and of out */
+  int32_t max_pages;    /* entries per page-table row */
+  int32_t reserved0;
+  int64_t n_pages;      /* pages in the pool (page ids are checked against it) */
+  const float* q;       /* [n][Hq][hd] float32, already rotated */
+  const void* pool;     /* KV pages */
+  const int32_t* page_table; /* [n][max_pages] */
+  const int32_t* lens;  /* [n] keys per row, 1..max_pages*page_size */
+  void* out;            /* [n][Hq*hd] in the dtype */
+  uint32_t* err;        /* optional device word: bit 1 = a bounded wait expired, bit 2 = bad page id */
+} tlf_attn_args;
+
+/* Scratch bytes tlf_attn_decode needs for these arguments on the current
+ * device (split-K work plan and partial results); 0 for invalid arguments. */
+size_t tlf_attn_decode_scratch_bytes(const tlf_attn_args* a);
+
+/* Launch the attention on `stream` (cudaStream_t) using caller-provided
+ * device scratch of at least tlf_attn_decode_scratch_bytes(a) bytes. Does not
+ * synchronise. Errors (INVALID_ARG, CUDA) are reported through
+ * tlf_last_error(NULL) on the calling thread. */
+int tlf_attn_decode(const tlf_attn_args* a, void* scratch, size_t scratch_bytes, void* stream);
+
 /* ---- inspection ---------------------------------------------------------- */
 
 /* Number of live sequences and free pages. */

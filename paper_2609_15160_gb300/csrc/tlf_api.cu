@@ -189,6 +189,11 @@ extern "C" int tlf_validate_config(const tlf_config* c, char* msg, size_t msg_le
   return TLF_OK;
 }
 
+int tlf::set_thread_error(int code, const char* msg) {
+  g_create_error = msg;
+  return code;
+}
+
 extern "C" int64_t tlf_page_bytes(const tlf_config* c) {
   if (tlf_validate_config(c, nullptr, 0) != TLF_OK) return 0;
   return page_bytes_of(*c);

@@ -12,6 +12,8 @@
 #include <cuda_runtime.h>
 #include <stdint.h>
 
+#include "tlf.h"
+
 namespace tlf {
 
 // ----------------------------------------------------------------------------
@@ -314,5 +316,18 @@ void launch_final(const ModelDims& md, const StepDev& s, int B, const float* gai
 void launch_scatter_cache(const ModelDims& md, int slot, int r, int n, const void* k, const void* v,
                           const int* positions, const int* page_table, void* pool, int* pos_table,
                           cudaStream_t st);
+
+// Kernel-level attention operation (tlf_attn_decode): scratch layout and launch.
+struct AttnOpLayout {
+  size_t m, slots, len, idx, count, item_base, nch, chunk, errw, part_o, part_ml, total;
+  int grid, target_items, items_max;
+};
+AttnOpLayout attn_op_layout(const tlf_attn_args* a, int num_sms);
+const char* attn_op_validate(const tlf_attn_args* a);
+cudaError_t attn_op_run(const tlf_attn_args* a, uint8_t* scratch, const AttnOpLayout& L, cudaStream_t st);
+int current_num_sms();
+
+// Record a message for tlf_last_error(NULL) on this thread; returns code.
+int set_thread_error(int code, const char* msg);
 
 }  // namespace tlf

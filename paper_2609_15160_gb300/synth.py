@@ -281,6 +281,34 @@ def make_cache_snapshot(m: ModelConfig, length: int, seed: int,
     return {"depths": np.asarray(depths, dtype=np.int32), "positions": pos, "k": ks, "v": vs}
 
 
+def make_attn_problem(n: int, lens, hq: int, hkv: int, hd: int, n_layers: int = 2, layer: int = 1,
+                      dtype: str = "bf16", seed: int = 0, spare_pages: int = 3, page_size: int = 64) -> dict:
+    """Inputs of the kernel-level attention operation on paged caches.
+
+    q [n, hq, hd] float32 (already rotated); pool [n_pages, J, 2, hkv, page, hd]
+    with values that are multiples of 1/64 in [-2, 2) (exact in bf16 and fp32);
+    page_table [n, max_pages] giving every row distinct, randomly placed pages.
+    """
+    rng = _rng(seed, 9)
+    lens = np.asarray(lens, dtype=np.int32)
+    if lens.size != n:
+        raise ValueError("one length per row")
+    need = [(int(L) + page_size - 1) // page_size for L in lens]
+    max_pages = max(need)
+    n_pages = sum(need) + spare_pages
+    perm = rng.permutation(n_pages)
+    pt = np.full((n, max_pages), -1, dtype=np.int32)
+    o = 0
+    for b in range(n):
+        pt[b, :need[b]] = perm[o:o + need[b]]
+        o += need[b]
+    pool = rng.integers(-128, 128, size=(n_pages, n_layers, 2, hkv, page_size, hd), dtype=np.int16)
+    pool = pool.astype(np.float32) / 64.0
+    q = rng.standard_normal((n, hq, hd), dtype=np.float32)
+    return dict(n=n, lens=lens, hq=hq, hkv=hkv, hd=hd, n_layers=n_layers, layer=layer, dtype=dtype,
+                q=q, pool=pool, page_table=pt, max_pages=max_pages, n_pages=n_pages, page_size=page_size)
+
+
 def expected_mean_depth(probs: Sequence[float]) -> float:
     return float(sum((i + 1) * p for i, p in enumerate(probs)))
 

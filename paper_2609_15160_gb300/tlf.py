@@ -39,6 +39,12 @@ class TlfWeights(C.Structure):
                                           "w_up", "w_down", "attn_norm", "mlp_norm", "final_norm")]
 
 
+class TlfAttnArgs(C.Structure):
+    _fields_ = [(n, C.c_int32) for n in ("n", "n_heads", "n_kv_heads", "head_dim", "n_layers", "layer",
+                                         "page_size", "dtype", "max_pages", "reserved0")] + [
+        ("n_pages", C.c_int64)] + [(n, C.c_void_p) for n in ("q", "pool", "page_table", "lens", "out", "err")]
+
+
 class TlfError(RuntimeError):
     def __init__(self, code: int, msg: str):
         super().__init__(f"{ERRORS.get(code, code)}: {msg}")
@@ -68,6 +74,8 @@ _SIGS = {
     "tlf_last_active_sets": (C.c_int, [_P, _I32P, _I32P]),
     "tlf_set_profiling": (C.c_int, [_P, C.c_int32]),
     "tlf_last_step_profile": (C.c_int, [_P, _F32P, C.POINTER(C.c_double), _I32P]),
+    "tlf_attn_decode_scratch_bytes": (C.c_size_t, [C.POINTER(TlfAttnArgs)]),
+    "tlf_attn_decode": (C.c_int, [C.POINTER(TlfAttnArgs), _P, C.c_size_t, _P]),
 }
 
 
@@ -195,6 +203,23 @@ def tlf_release(ctx, seq_id: int):
 def tlf_load_cache(ctx, seq_id: int, lens: np.ndarray, positions: np.ndarray, k: np.ndarray, v: np.ndarray):
     _check(load_library().tlf_load_cache(ctx, C.c_uint64(seq_id), _ptr(lens, C.c_int32), _ptr(positions, C.c_int32),
                                          k.ctypes.data, v.ctypes.data), ctx)
+
+
+def attn_args(n, n_heads, n_kv_heads, head_dim, n_layers, layer, dtype, max_pages, n_pages, q, pool, page_table,
+              lens, out, err=None) -> TlfAttnArgs:
+    """Arguments of tlf_attn_decode; buffers are torch CUDA tensors (or raw device addresses)."""
+    return TlfAttnArgs(n=n, n_heads=n_heads, n_kv_heads=n_kv_heads, head_dim=head_dim, n_layers=n_layers,
+                       layer=layer, page_size=64, dtype=DTYPE[dtype] if isinstance(dtype, str) else dtype,
+                       max_pages=max_pages, reserved0=0, n_pages=n_pages, q=_addr(q), pool=_addr(pool),
+                       page_table=_addr(page_table), lens=_addr(lens), out=_addr(out), err=_addr(err))
+
+
+def tlf_attn_decode_scratch_bytes(a: TlfAttnArgs) -> int:
+    return load_library().tlf_attn_decode_scratch_bytes(C.byref(a))
+
+
+def tlf_attn_decode(a: TlfAttnArgs, scratch, scratch_bytes: int, stream=None):
+    _check(load_library().tlf_attn_decode(C.byref(a), _addr(scratch), scratch_bytes, _stream(stream)), None)
 
 
 # ----------------------------------------------------------------------------
