@@ -233,6 +233,24 @@ size_t tlf_attn_decode_scratch_bytes(const tlf_attn_args* a);
  * tlf_last_error(NULL) on the calling thread. */
 int tlf_attn_decode(const tlf_attn_args* a, void* scratch, size_t scratch_bytes, void* stream);
 
+/* The same attention as tlf_attn_decode, for callers that cannot allocate
+ * device memory: for instance a plug-in whose host application owns every
+ * byte of the GPU through its own pool, or a request path where a
+ * cudaMalloc (which can synchronise the device and stall other work) is not
+ * allowed. It allocates nothing; its scratch is a 4 MiB array built into the
+ * library, present on every GPU that loads the library until the process
+ * exits. Arguments whose scratch (tlf_attn_decode_scratch_bytes) exceeds
+ * 4 MiB are rejected with TLF_ERR_INVALID_ARG and a message naming the
+ * sizes; a C4-shaped call (16 rows, Hq 16 / Hkv 8, hd 128) needs under 1
+ * MiB. The first call on a device looks up the array's device address (a
+ * set-up step), so make that first call before any stream capture. Every
+ * call on a device shares the array and it keeps the last call's contents:
+ * calls whose kernels overlap on the GPU (different streams, or other host
+ * threads) race and must not be issued; serialise them. Launches on
+ * `stream` without synchronising; errors as for tlf_attn_decode. The paper
+ * has no counterpart of this entry point. */
+int tlf_attn_decode_static(const tlf_attn_args* a, void* stream);
+
 /* ---- inspection ---------------------------------------------------------- */
 
 /* Number of live sequences and free pages. */

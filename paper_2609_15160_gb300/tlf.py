@@ -76,6 +76,7 @@ _SIGS = {
     "tlf_last_step_profile": (C.c_int, [_P, _F32P, C.POINTER(C.c_double), _I32P]),
     "tlf_attn_decode_scratch_bytes": (C.c_size_t, [C.POINTER(TlfAttnArgs)]),
     "tlf_attn_decode": (C.c_int, [C.POINTER(TlfAttnArgs), _P, C.c_size_t, _P]),
+    "tlf_attn_decode_static": (C.c_int, [C.POINTER(TlfAttnArgs), _P]),
 }
 
 
@@ -220,6 +221,11 @@ def tlf_attn_decode_scratch_bytes(a: TlfAttnArgs) -> int:
 
 def tlf_attn_decode(a: TlfAttnArgs, scratch, scratch_bytes: int, stream=None):
     _check(load_library().tlf_attn_decode(C.byref(a), _addr(scratch), scratch_bytes, _stream(stream)), None)
+
+
+def tlf_attn_decode_static(a: TlfAttnArgs, stream=None):
+    """tlf_attn_decode without caller scratch: uses the library's built-in 4 MiB device array."""
+    _check(load_library().tlf_attn_decode_static(C.byref(a), _stream(stream)), None)
 
 
 # ----------------------------------------------------------------------------
