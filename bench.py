@@ -167,13 +167,13 @@ def run_reference(args):
     print(json.dumps(line))
 
 
-def setup_workload(T, wl, rank: int, gemm_impl="auto", prefill="auto"):
+def setup_workload(T, wl, rank: int, gemm_impl="auto", prefill="auto", extra_tokens: int = 0):
     m = wl.model
     w = synth.make_weights(m)
     B = wl.batch
     prompts = synth.make_prompts(wl)
     lengths = [len(p) for p in prompts]
-    steps_cap = wl.decode_steps + 64
+    steps_cap = max(wl.decode_steps, extra_tokens) + 64
     use_snapshot = prefill == "snapshot" or (prefill == "auto" and max(lengths) > 4096)
     ids = [rank * 100000 + b for b in range(B)]
     if use_snapshot:
@@ -217,7 +217,8 @@ def run_ours(args):
     m = wl.model
     B = wl.batch
     t0 = time.time()
-    ctx, ids, how = setup_workload(T, wl, rank, prefill=args.prefill)
+    ctx, ids, how = setup_workload(T, wl, rank, prefill=args.prefill,
+                                   extra_tokens=3 * (args.warmup + args.steps))
     setup_s = time.time() - t0
     stream = torch.cuda.current_stream()
     n_steps = args.warmup + args.steps
@@ -372,8 +373,8 @@ def main():
     ap.add_argument("--batch", type=int, default=16)
     ap.add_argument("--context", type=int, default=32768)
     ap.add_argument("--gpus", type=int, default=1)
-    ap.add_argument("--steps", type=int, default=32)
-    ap.add_argument("--warmup", type=int, default=5)
+    ap.add_argument("--steps", type=int, default=100)
+    ap.add_argument("--warmup", type=int, default=10)
     ap.add_argument("--config", default="c4", choices=sorted(DESCR))
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--prefill", default="auto", choices=["auto", "snapshot", "real"])

@@ -56,6 +56,8 @@ __global__ void __launch_bounds__(256) k_attn_decode(ModelDims md, StepDev s, in
   float* red = reinterpret_cast<float*>(ring + S::NST * S::STAGE_BYTES);  // [warps][G][HD + 2]
   uint64_t* bars = reinterpret_cast<uint64_t*>(red + ATT_WARPS * G * (HD + 2));
 
+  pdl_wait();
+  pdl_trigger();
   const int n_r = s.n[r];
   const int items = s.item_base[r * (md.max_batch + 1) + n_r];
   if ((int)blockIdx.x >= items) return;
@@ -257,6 +259,8 @@ __global__ void __launch_bounds__(256) k_attn_decode(ModelDims md, StepDev s, in
 template <typename T, int HD, int G>
 __global__ void __launch_bounds__(128) k_attn_combine(ModelDims md, StepDev s, int r, const float* __restrict__ part_o,
                                                       const float* __restrict__ part_ml, T* __restrict__ O) {
+  pdl_wait();
+  pdl_trigger();
   const int k = blockIdx.x, h = blockIdx.y;
   if (k >= s.n[r]) return;
   const int kvh = h / G, g = h % G;
@@ -285,14 +289,14 @@ static void attn_launch(const ModelDims& md, const StepDev& s, int r, int j, con
     cudaFuncSetAttribute(k_attn_decode<T, HD, G>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
     attr = true;
   }
-  k_attn_decode<T, HD, G><<<grid, 32 * ATT_WARPS, smem, st>>>(md, s, r, j, Q, po, pml);
+  launch_k(k_attn_decode<T, HD, G>, grid, 32 * ATT_WARPS, smem, st, md, s, r, j, Q, po, pml);
 }
 
 template <typename T, int HD, int G>
 static void combine_launch(const ModelDims& md, const StepDev& s, int r, const float* po, const float* pml, void* O,
                            cudaStream_t st) {
   dim3 grid(md.max_batch, md.Hq);
-  k_attn_combine<T, HD, G><<<grid, HD < 128 ? HD : 128, 0, st>>>(md, s, r, po, pml, (T*)O);
+  launch_k(k_attn_combine<T, HD, G>, grid, HD < 128 ? HD : 128, 0, st, md, s, r, po, pml, (T*)O);
 }
 
 #define TLF_ATTN_DISPATCH(FN, ...)                                                              \

@@ -60,8 +60,15 @@ __global__ void __launch_bounds__(128) k_gemm_tc(const __grid_constant__ CUtenso
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 2 * TC_STAGES + 1);
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int n = a.n_dev ? *a.n_dev : a.n_host;
-  if (n <= 0) return;
+  // The token count comes from the plan kernel, which completed before this
+  // grid was launched (every kernel triggers its successor only after its own
+  // wait), so it is read before pdl_wait(), bypassing L1.
+  const int n = a.n_dev ? __ldcg(a.n_dev) : a.n_host;
+  if (n <= 0) {
+    pdl_wait();
+    pdl_trigger();
+    return;
+  }
   const int ncols = ((n + 15) / 16) * 16;  // MMA N: multiple of 16, <= NT
   const int m0 = blockIdx.x * TC_BM;
   const int split = blockIdx.y;
@@ -93,19 +100,32 @@ __global__ void __launch_bounds__(128) k_gemm_tc(const __grid_constant__ CUtenso
   tc_fence_after();
   const uint32_t tmem = *tmem_slot;
 
+  if (warp == 0 && lane == 0) {
+    // TMA producer. Weight tiles of the first stages go out before the wait on
+    // the preceding kernels (weights are never written by them); token tiles after.
+    const int pre = nk < TC_STAGES ? nk : TC_STAGES;
+    for (int i = 0; i < pre; ++i) {
+      mbar_arrive_expect_tx(full(i), A_BYTES + B_BYTES);
+      tma_load_2d(smem_u32(sA + i * A_BYTES), &mapW, (kb0 + i) * TC_BK, m0, full(i));
+    }
+    pdl_wait();
+    pdl_trigger();
+    for (int i = 0; i < pre; ++i) tma_load_2d(smem_u32(sB + i * B_BYTES), &mapX, (kb0 + i) * TC_BK, 0, full(i));
+    for (int i = pre; i < nk; ++i) {
+      const int st = i % TC_STAGES;
+      const uint32_t ph = (uint32_t)(i / TC_STAGES) & 1u;
+      if (!mbar_wait(empty(st), ph ^ 1u, a.err)) break;
+      mbar_arrive_expect_tx(full(st), A_BYTES + B_BYTES);
+      const int kx = (kb0 + i) * TC_BK;
+      tma_load_2d(smem_u32(sA + st * A_BYTES), &mapW, kx, m0, full(st));
+      tma_load_2d(smem_u32(sB + st * B_BYTES), &mapX, kx, 0, full(st));
+    }
+  } else {
+    pdl_wait();
+    pdl_trigger();
+  }
   if (nk > 0) {
-    if (warp == 0 && lane == 0) {
-      // TMA producer
-      for (int i = 0; i < nk; ++i) {
-        const int st = i % TC_STAGES;
-        const uint32_t ph = (uint32_t)(i / TC_STAGES) & 1u;
-        if (!mbar_wait(empty(st), ph ^ 1u, a.err)) break;
-        mbar_arrive_expect_tx(full(st), A_BYTES + B_BYTES);
-        const int kx = (kb0 + i) * TC_BK;
-        tma_load_2d(smem_u32(sA + st * A_BYTES), &mapW, kx, m0, full(st));
-        tma_load_2d(smem_u32(sB + st * B_BYTES), &mapX, kx, 0, full(st));
-      }
-    } else if (warp == 1 && lane == 0) {
+    if (warp == 1 && lane == 0) {
       // MMA issuer
       const uint32_t idesc = idesc_bf16_f32(TC_BM, ncols);
       for (int i = 0; i < nk; ++i) {
@@ -163,7 +183,7 @@ static void launch_tc_nt(const CUtensorMap* mapW, const CUtensorMap* mapX, const
     attr_set = true;
   }
   dim3 grid((a.N + TC_BM - 1) / TC_BM, a.splits);
-  k_gemm_tc<NT><<<grid, 128, smem, st>>>(*mapW, *mapX, a);
+  launch_k(k_gemm_tc<NT>, grid, 128, smem, st, *mapW, *mapX, a);
 }
 
 void launch_gemm_tc(const CUtensorMap* mapW, const CUtensorMap* mapX, int nt_max, const GemmArgs& a,
@@ -185,6 +205,8 @@ __global__ void __launch_bounds__(256) k_gemm_simt(const T* __restrict__ W, cons
                                                    GemmArgs a) {
   __shared__ float Ws[32][65];
   __shared__ float Xs[32][33];
+  pdl_wait();
+  pdl_trigger();
   const int n = a.n_dev ? *a.n_dev : a.n_host;
   if (n <= 0) return;
   const int f0 = blockIdx.x * 64;
@@ -234,9 +256,9 @@ __global__ void __launch_bounds__(256) k_gemm_simt(const T* __restrict__ W, cons
 void launch_gemm_simt(int dtype, const void* W, const void* X, int ldx, const GemmArgs& a, cudaStream_t st) {
   dim3 grid((a.N + 63) / 64, a.splits);
   if (dtype == 1)
-    k_gemm_simt<bf16><<<grid, 256, 0, st>>>((const bf16*)W, (const bf16*)X, ldx, a);
+    launch_k(k_gemm_simt<bf16>, grid, 256, 0, st, (const bf16*)W, (const bf16*)X, ldx, a);
   else
-    k_gemm_simt<float><<<grid, 256, 0, st>>>((const float*)W, (const float*)X, ldx, a);
+    launch_k(k_gemm_simt<float>, grid, 256, 0, st, (const float*)W, (const float*)X, ldx, a);
 }
 
 }  // namespace tlf

@@ -32,33 +32,63 @@ __global__ void __launch_bounds__(256) k_norm_rows(const float* __restrict__ H, 
                                                    const int* __restrict__ n_dev, int n_host,
                                                    const float* __restrict__ gain, int d, float eps,
                                                    T* __restrict__ X, int ldx) {
+  pdl_wait();
+  pdl_trigger();
   const int k = blockIdx.x;
   const int n = n_dev ? *n_dev : n_host;
   if (k >= n) return;
   const int src = idx ? idx[k] : k;
-  const float* h = H + (size_t)src * ldh;
+  // the row (d <= 8192, a multiple of 64) is read once into registers, 16 bytes per load
+  const float4* h4 = reinterpret_cast<const float4*>(H + (size_t)src * ldh);
+  const float4* g4 = reinterpret_cast<const float4*>(gain);
+  const int d4 = d / 4;
+  float4 v[8];
   float ss = 0.f;
-  for (int i = threadIdx.x; i < d; i += blockDim.x) ss += h[i] * h[i];
+#pragma unroll
+  for (int c = 0; c < 8; ++c) {
+    const int i = threadIdx.x + c * blockDim.x;
+    if (i < d4) {
+      v[c] = h4[i];
+      ss += v[c].x * v[c].x + v[c].y * v[c].y + v[c].z * v[c].z + v[c].w * v[c].w;
+    }
+  }
   ss = block_sum(ss);
   const float inv = rsqrtf(ss / (float)d + eps);
-  for (int i = threadIdx.x; i < d; i += blockDim.x) X[(size_t)k * ldx + i] = from_f32<T>(h[i] * inv * gain[i]);
+  T* xr = X + (size_t)k * ldx;
+#pragma unroll
+  for (int c = 0; c < 8; ++c) {
+    const int i = threadIdx.x + c * blockDim.x;
+    if (i < d4) {
+      const float4 g = g4[i];
+      xr[4 * i + 0] = from_f32<T>(v[c].x * inv * g.x);
+      xr[4 * i + 1] = from_f32<T>(v[c].y * inv * g.y);
+      xr[4 * i + 2] = from_f32<T>(v[c].z * inv * g.z);
+      xr[4 * i + 3] = from_f32<T>(v[c].w * inv * g.w);
+    }
+  }
 }
 
 void launch_norm_rows(int dtype, const float* H, int ldh, const int* idx, const int* n_dev, int n_host, int rows_max,
                       const float* gain, int d, float eps, void* X, int ldx, cudaStream_t st) {
   if (rows_max <= 0) return;
   if (dtype == 1)
-    k_norm_rows<bf16><<<rows_max, 256, 0, st>>>(H, ldh, idx, n_dev, n_host, gain, d, eps, (bf16*)X, ldx);
+    launch_k(k_norm_rows<bf16>, rows_max, 256, 0, st, H, ldh, idx, n_dev, n_host, gain, d, eps, (bf16*)X, ldx);
   else
-    k_norm_rows<float><<<rows_max, 256, 0, st>>>(H, ldh, idx, n_dev, n_host, gain, d, eps, (float*)X, ldx);
+    launch_k(k_norm_rows<float>, rows_max, 256, 0, st, H, ldh, idx, n_dev, n_host, gain, d, eps, (float*)X, ldx);
 }
 
 template <typename T>
 __global__ void __launch_bounds__(256) k_rope_append(ModelDims md, StepDev s, int r, int j,
                                                      const float* __restrict__ part, int splits, float* __restrict__ Q,
                                                      const double* __restrict__ inv_freq) {
+  pdl_wait();
+  pdl_trigger();
   const int k = blockIdx.x;
   if (k >= s.n[r]) return;
+  const int hd2 = md.hd / 2;
+  const int n_pairs = (md.Hq + md.Hkv) * hd2;   // rotated q and k pairs, then v elements
+  const int t = blockIdx.y * blockDim.x + threadIdx.x;
+  if (t >= n_pairs + md.Hkv * md.hd) return;
   const int b = s.idx[r * md.max_batch + k];
   const int slot = s.slots[b];
   const int pos = s.len[slot * md.M + 0];  // every token runs loop 1: its length is the token count
@@ -66,7 +96,7 @@ __global__ void __launch_bounds__(256) k_rope_append(ModelDims md, StepDev s, in
   const int ps = md.page_size, hd = md.hd, half = hd / 2;
   const int page = s.page_table[((size_t)slot * md.M + r) * md.max_pages + L / ps];
   if (page < 0 || page >= md.n_pages) {
-    if (threadIdx.x == 0) atomicOr(s.err, DEVERR_INDEX);
+    if (t == 0) atomicOr(s.err, DEVERR_INDEX);
     return;
   }
   const int off = L % ps;
@@ -75,8 +105,8 @@ __global__ void __launch_bounds__(256) k_rope_append(ModelDims md, StepDev s, in
   const float* prow = part + (size_t)k * md.qkv_dim;
   const double two_pi = 6.283185307179586476925286766559;
 
-  // q heads then k heads: rotate pair (i, i + hd/2) by pos * theta_i
-  for (int t = threadIdx.x; t < (md.Hq + md.Hkv) * half; t += blockDim.x) {
+  if (t < n_pairs) {
+    // q heads then k heads: rotate pair (i, i + hd/2) by pos * theta_i
     const int h = t / half, i = t % half;
     const int c0 = h * hd + i, c1 = c0 + half;  // k columns follow the q columns
     float a = 0.f, c = 0.f;
@@ -98,29 +128,33 @@ __global__ void __launch_bounds__(256) k_rope_append(ModelDims md, StepDev s, in
       kp[i] = from_f32<T>(ra);
       kp[i + half] = from_f32<T>(rc);
     }
-  }
-  for (int t = threadIdx.x; t < md.Hkv * hd; t += blockDim.x) {
-    const int h = t / hd, e = t % hd;
-    const int col = md.q_dim + md.kv_dim + t;
+  } else {
+    const int tv = t - n_pairs;
+    const int h = tv / hd, e = tv % hd;
+    const int col = md.q_dim + md.kv_dim + tv;
     float a = 0.f;
     for (int sp = 0; sp < splits; ++sp) a += prow[sp * pstride + col];
     T* vp = pg + ((size_t)(j * 2 + 1) * md.Hkv + h) * ps * hd + (size_t)off * hd;
     vp[e] = from_f32<T>(a);
   }
-  if (j == 0 && threadIdx.x == 0) s.pos_table[(size_t)page * ps + off] = pos;
+  if (j == 0 && t == 0) s.pos_table[(size_t)page * ps + off] = pos;
 }
 
 void launch_rope_append(const ModelDims& md, const StepDev& s, int r, int j, const float* part, int splits, float* Q,
                         const double* inv_freq, cudaStream_t st) {
+  const int work = (md.Hq + md.Hkv) * (md.hd / 2) + md.Hkv * md.hd;
+  dim3 grid(md.max_batch, (work + 127) / 128);
   if (md.dtype == 1)
-    k_rope_append<bf16><<<md.max_batch, 256, 0, st>>>(md, s, r, j, part, splits, Q, inv_freq);
+    launch_k(k_rope_append<bf16>, grid, 128, 0, st, md, s, r, j, part, splits, Q, inv_freq);
   else
-    k_rope_append<float><<<md.max_batch, 256, 0, st>>>(md, s, r, j, part, splits, Q, inv_freq);
+    launch_k(k_rope_append<float>, grid, 128, 0, st, md, s, r, j, part, splits, Q, inv_freq);
 }
 
 template <typename T>
 __global__ void __launch_bounds__(256) k_swiglu(const float* __restrict__ part, int splits, int max_rows,
                                                 const int* __restrict__ n_dev, int ff, T* __restrict__ U) {
+  pdl_wait();
+  pdl_trigger();
   const int k = blockIdx.y;
   if (k >= *n_dev) return;
   const size_t N = 2 * (size_t)ff;
@@ -139,14 +173,16 @@ void launch_swiglu(int dtype, const float* part, int splits, int max_rows, const
                    cudaStream_t st) {
   dim3 grid((ff + 255) / 256, max_rows);
   if (dtype == 1)
-    k_swiglu<bf16><<<grid, 256, 0, st>>>(part, splits, max_rows, n_dev, ff, (bf16*)U);
+    launch_k(k_swiglu<bf16>, grid, 256, 0, st, part, splits, max_rows, n_dev, ff, (bf16*)U);
   else
-    k_swiglu<float><<<grid, 256, 0, st>>>(part, splits, max_rows, n_dev, ff, (float*)U);
+    launch_k(k_swiglu<float>, grid, 256, 0, st, part, splits, max_rows, n_dev, ff, (float*)U);
 }
 
 template <typename T>
 __global__ void __launch_bounds__(256) k_final(ModelDims md, StepDev s, const float* __restrict__ gain,
                                                T* __restrict__ Xf) {
+  pdl_wait();
+  pdl_trigger();
   const int b = blockIdx.x;
   const float* h = s.H + (size_t)b * md.d;
   float ss = 0.f;
@@ -162,9 +198,9 @@ __global__ void __launch_bounds__(256) k_final(ModelDims md, StepDev s, const fl
 
 void launch_final(const ModelDims& md, const StepDev& s, int B, const float* gain, void* Xf, cudaStream_t st) {
   if (md.dtype == 1)
-    k_final<bf16><<<B, 256, 0, st>>>(md, s, gain, (bf16*)Xf);
+    launch_k(k_final<bf16>, B, 256, 0, st, md, s, gain, (bf16*)Xf);
   else
-    k_final<float><<<B, 256, 0, st>>>(md, s, gain, (float*)Xf);
+    launch_k(k_final<float>, B, 256, 0, st, md, s, gain, (float*)Xf);
 }
 
 // Snapshot entries e < n of loop r: src layout [n][J][Hkv][hd] for k and v.

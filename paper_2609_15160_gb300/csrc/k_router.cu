@@ -18,7 +18,10 @@ namespace tlf {
 template <typename T>
 __global__ void __launch_bounds__(256) k_router(ModelDims md, StepDev s, int B, const T* __restrict__ emb,
                                                 const T* __restrict__ rw, const float* __restrict__ rb,
-                                                const PageUpdate* __restrict__ upd, int n_upd) {
+                                                const PageUpdate* __restrict__ upd, const int* __restrict__ n_upd_dev) {
+  pdl_wait();
+  pdl_trigger();
+  const int n_upd = *n_upd_dev;
   for (int u = blockIdx.x * blockDim.x + threadIdx.x; u < n_upd; u += gridDim.x * blockDim.x) {
     const PageUpdate p = upd[u];
     s.page_table[p.index] = p.page;
@@ -137,6 +140,8 @@ __device__ int block_exclusive_scan(int v, int* total) {
 }
 
 __global__ void __launch_bounds__(256) k_plan(ModelDims md, StepDev s, int B, int target_items, int min_chunk) {
+  pdl_wait();
+  pdl_trigger();
   const int b = threadIdx.x;
   const int lane = b & 31;
   const int mb = (b < B) ? s.m[b] : 0;
@@ -174,17 +179,18 @@ __global__ void __launch_bounds__(256) k_plan(ModelDims md, StepDev s, int B, in
 }
 
 void launch_router(const ModelDims& md, const StepDev& s, int B, const void* emb, const void* router_w,
-                   const float* router_b, const PageUpdate* upd, int n_upd, cudaStream_t st) {
+                   const float* router_b, const PageUpdate* upd, const int* n_upd, cudaStream_t st) {
   const int grid = (B + 7) / 8;
   if (md.dtype == 1)
-    k_router<bf16><<<grid, 256, 0, st>>>(md, s, B, (const bf16*)emb, (const bf16*)router_w, router_b, upd, n_upd);
+    launch_k(k_router<bf16>, grid, 256, 0, st, md, s, B, (const bf16*)emb, (const bf16*)router_w, router_b, upd,
+             n_upd);
   else
-    k_router<float><<<grid, 256, 0, st>>>(md, s, B, (const float*)emb, (const float*)router_w, router_b, upd,
-                                          n_upd);
+    launch_k(k_router<float>, grid, 256, 0, st, md, s, B, (const float*)emb, (const float*)router_w, router_b, upd,
+             n_upd);
 }
 
 void launch_plan(const ModelDims& md, const StepDev& s, int B, int target_items, int min_chunk, cudaStream_t st) {
-  k_plan<<<1, 256, 0, st>>>(md, s, B, target_items, min_chunk);
+  launch_k(k_plan, 1, 256, 0, st, md, s, B, target_items, min_chunk);
 }
 
 }  // namespace tlf

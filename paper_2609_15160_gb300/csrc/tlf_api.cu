@@ -113,7 +113,20 @@ struct tlf_ctx {
   double last_attn_bytes = 0.0;
   int last_launches = 0;
   std::vector<cudaEvent_t> events;
+  int n_events = 0;
   int last_batch = 0;
+
+  // CUDA graphs of the step
+  struct StepGraph {
+    int B;
+    bool logits;
+    cudaGraphExec_t exec;
+    int launches;
+  };
+  std::vector<StepGraph> graphs;
+  cudaStream_t cap_stream = nullptr;
+  bool use_graphs = true;
+  bool warmed = false;
 };
 
 // ----------------------------------------------------------------------------
@@ -160,7 +173,7 @@ extern "C" int tlf_validate_config(const tlf_config* c, char* msg, size_t msg_le
   if (!c) return bad("config is NULL");
   if (c->dtype != TLF_DTYPE_F32 && c->dtype != TLF_DTYPE_BF16) return bad("dtype must be TLF_DTYPE_F32 or TLF_DTYPE_BF16");
   if (c->vocab < 1) return bad("vocab must be >= 1");
-  if (c->d_model < 64 || c->d_model % 64) return bad("d_model must be a positive multiple of 64");
+  if (c->d_model < 64 || c->d_model % 64 || c->d_model > 8192) return bad("d_model must be a multiple of 64 in 64..8192");
   if (c->n_heads < 1 || c->n_kv_heads < 1 || c->n_heads % c->n_kv_heads) return bad("n_kv_heads must divide n_heads");
   const int g = c->n_heads / c->n_kv_heads;
   if (!(g == 1 || g == 2 || (g == 4 && c->dtype == TLF_DTYPE_BF16 && c->head_dim >= 64)))
@@ -188,6 +201,12 @@ extern "C" int tlf_validate_config(const tlf_config* c, char* msg, size_t msg_le
   if (msg && msg_len) snprintf(msg, msg_len, "ok");
   return TLF_OK;
 }
+
+// Programmatic dependent launch for the step kernels (TLF_NO_PDL=1 turns it off).
+bool tlf::g_use_pdl = [] {
+  const char* e = getenv("TLF_NO_PDL");
+  return !(e && e[0] == '1');
+}();
 
 int tlf::set_thread_error(int code, const char* msg) {
   g_create_error = msg;
@@ -415,6 +434,11 @@ static int create_impl(tlf_ctx* ctx, const tlf_weights* w) {
   CK(ctx, cudaMallocHost((void**)&ctx->h_m, (size_t)B * 4));
   CK(ctx, cudaMallocHost((void**)&ctx->h_margin, (size_t)B * 4));
   CK(ctx, cudaMallocHost((void**)&ctx->h_err, 16));
+  CK(ctx, cudaStreamCreateWithFlags(&ctx->cap_stream, cudaStreamNonBlocking));
+  {
+    const char* e = getenv("TLF_NO_GRAPH");
+    ctx->use_graphs = !(e && e[0] == '1');
+  }
   ctx->events.resize(2 * M * J + 2);
   for (auto& e : ctx->events) CK(ctx, cudaEventCreate(&e));
   CK(ctx, cudaDeviceSynchronize());
@@ -439,6 +463,8 @@ extern "C" void tlf_destroy(tlf_ctx* ctx) {
     if (ctx->h_margin) cudaFreeHost(ctx->h_margin);
     if (ctx->h_err) cudaFreeHost(ctx->h_err);
     for (auto e : ctx->events) if (e) cudaEventDestroy(e);
+    for (auto& g : ctx->graphs) cudaGraphExecDestroy(g.exec);
+    if (ctx->cap_stream) cudaStreamDestroy(ctx->cap_stream);
   }
   delete ctx;
 }
@@ -553,24 +579,19 @@ static void gemm(tlf_ctx* ctx, const DeviceMat& W, const CUtensorMap* xmap, cons
   ++ctx->last_launches;
 }
 
-static int run_step(tlf_ctx* ctx, int B, const int* slots, const int* tokens, const int* forced,
-                    const std::vector<PageUpdate>& upd, bool need_logits, cudaStream_t st) {
+// All device work of one step on `st`: upload of the step inputs from the pinned
+// buffer, every kernel, and the download of loop counts, margins and the error
+// word. Capturable in a CUDA graph (nothing here depends on host values that
+// change between steps with the same batch size).
+static int enqueue_step(tlf_ctx* ctx, int B, bool need_logits, bool prof, cudaStream_t st) {
   const ModelDims& md = ctx->md;
   const int M = md.M, J = md.J, maxB = md.max_batch;
-  int* h = ctx->h_upload;
-  for (int b = 0; b < B; ++b) {
-    h[b] = tokens[b];
-    h[B + b] = forced ? forced[b] : -1;
-    h[2 * B + b] = slots[b];
-  }
-  const size_t nu = upd.size();
-  memcpy(h + 3 * B, upd.data(), nu * sizeof(PageUpdate));
-  CK(ctx, cudaMemcpyAsync(ctx->d_upload, h, (3 * B + 2 * nu) * 4, cudaMemcpyHostToDevice, st));
+  CK(ctx, cudaMemcpyAsync(ctx->d_upload, ctx->h_upload, ctx->upload_ints * 4, cudaMemcpyHostToDevice, st));
 
   StepDev s{};
-  s.tokens = ctx->d_upload;
-  s.forced = ctx->d_upload + B;
-  s.slots = ctx->d_upload + 2 * B;
+  s.tokens = ctx->d_upload + 1;
+  s.forced = ctx->d_upload + 1 + B;
+  s.slots = ctx->d_upload + 1 + 2 * B;
   s.m = ctx->d_m;
   s.margin = ctx->d_margin;
   s.H = ctx->d_H;
@@ -584,13 +605,12 @@ static int run_step(tlf_ctx* ctx, int B, const int* slots, const int* tokens, co
   s.pos_table = ctx->d_pos_table;
   s.pool = ctx->d_pool;
   s.err = ctx->d_err;
-  const PageUpdate* d_upd = reinterpret_cast<const PageUpdate*>(ctx->d_upload + 3 * B);
+  const PageUpdate* d_upd = reinterpret_cast<const PageUpdate*>(ctx->d_upload + 1 + 3 * B);
 
   ctx->last_launches = 0;
-  launch_router(md, s, B, ctx->d_emb, ctx->d_router_w, ctx->d_router_b, d_upd, (int)nu, st);
+  launch_router(md, s, B, ctx->d_emb, ctx->d_router_w, ctx->d_router_b, d_upd, ctx->d_upload, st);
   launch_plan(md, s, B, ctx->attn_target_items, ctx->attn_min_chunk, st);
   ctx->last_launches += 2;
-  const bool prof = ctx->profiling;
   int ev = 0;
   for (int r = 0; r < M; ++r) {
     const int* n_dev = ctx->d_n + r;
@@ -643,6 +663,7 @@ static int run_step(tlf_ctx* ctx, int B, const int* slots, const int* tokens, co
   }
   launch_final(md, s, B, ctx->d_final_norm, ctx->d_Xf, st);
   ++ctx->last_launches;
+  ctx->n_events = ev;
   if (need_logits) {
     GemmArgs a{};
     a.n_host = B;
@@ -657,6 +678,60 @@ static int run_step(tlf_ctx* ctx, int B, const int* slots, const int* tokens, co
   CK(ctx, cudaMemcpyAsync(ctx->h_m, ctx->d_m, (size_t)B * 4, cudaMemcpyDeviceToHost, st));
   CK(ctx, cudaMemcpyAsync(ctx->h_margin, ctx->d_margin, (size_t)B * 4, cudaMemcpyDeviceToHost, st));
   CK(ctx, cudaMemcpyAsync(ctx->h_err, ctx->d_err, 4, cudaMemcpyDeviceToHost, st));
+  return TLF_OK;
+}
+
+// The step as one CUDA graph per (batch size, logits on/off), built on first
+// use after the kernels have run once directly (their attributes are set).
+static cudaGraphExec_t step_graph(tlf_ctx* ctx, int B, bool need_logits) {
+  for (auto& g : ctx->graphs)
+    if (g.B == B && g.logits == need_logits) {
+      ctx->last_launches = g.launches;
+      return g.exec;
+    }
+  if (!ctx->use_graphs || !ctx->warmed || ctx->graphs.size() >= 32) return nullptr;
+  cudaGraph_t graph = nullptr;
+  cudaGraphExec_t exec = nullptr;
+  if (cudaStreamBeginCapture(ctx->cap_stream, cudaStreamCaptureModeThreadLocal) != cudaSuccess) {
+    cudaGetLastError();
+    ctx->use_graphs = false;
+    return nullptr;
+  }
+  const int rc = enqueue_step(ctx, B, need_logits, false, ctx->cap_stream);
+  const cudaError_t e1 = cudaStreamEndCapture(ctx->cap_stream, &graph);
+  if (rc != TLF_OK || e1 != cudaSuccess || cudaGraphInstantiate(&exec, graph, 0) != cudaSuccess) {
+    cudaGetLastError();
+    if (graph) cudaGraphDestroy(graph);
+    ctx->use_graphs = false;  // run the kernels directly from now on
+    return nullptr;
+  }
+  cudaGraphDestroy(graph);
+  ctx->graphs.push_back({B, need_logits, exec, ctx->last_launches});
+  return exec;
+}
+
+static int run_step(tlf_ctx* ctx, int B, const int* slots, const int* tokens, const int* forced,
+                    const std::vector<PageUpdate>& upd, bool need_logits, cudaStream_t st) {
+  const ModelDims& md = ctx->md;
+  const int M = md.M, J = md.J;
+  const bool prof = ctx->profiling;
+  int* h = ctx->h_upload;
+  const size_t nu = upd.size();
+  h[0] = (int)nu;
+  for (int b = 0; b < B; ++b) {
+    h[1 + b] = tokens[b];
+    h[1 + B + b] = forced ? forced[b] : -1;
+    h[1 + 2 * B + b] = slots[b];
+  }
+  memcpy(h + 1 + 3 * B, upd.data(), nu * sizeof(PageUpdate));
+  cudaGraphExec_t exec = prof ? nullptr : step_graph(ctx, B, need_logits);
+  if (exec) {
+    CK(ctx, cudaGraphLaunch(exec, st));
+  } else {
+    const int rc = enqueue_step(ctx, B, need_logits, prof, st);
+    if (rc) return rc;
+    ctx->warmed = true;
+  }
   CK(ctx, cudaStreamSynchronize(st));
   if (*ctx->h_err) {
     const uint32_t e = *ctx->h_err;
@@ -665,7 +740,7 @@ static int run_step(tlf_ctx* ctx, int B, const int* slots, const int* tokens, co
   }
   if (prof) {
     float tot = 0.f;
-    for (int i = 0; i + 1 < ev; i += 2) {
+    for (int i = 0; i + 1 < ctx->n_events; i += 2) {
       float ms = 0.f;
       cudaEventElapsedTime(&ms, ctx->events[i], ctx->events[i + 1]);
       tot += ms;

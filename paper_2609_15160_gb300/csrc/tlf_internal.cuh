@@ -28,6 +28,35 @@ enum : uint32_t {
 constexpr uint64_t kWaitLimitNs = 4000000000ull;  // 4 s
 
 // ----------------------------------------------------------------------------
+// Programmatic dependent launch. Every kernel of the step is launched with
+// programmatic stream serialisation: it may start while its predecessor in the
+// stream is still running, does work that reads nothing the predecessors write
+// (barrier set-up, TMEM allocation, weight tiles), then waits for them with
+// pdl_wait() and lets its own successor start with pdl_trigger(). Without the
+// launch attribute both instructions are no-ops.
+// ----------------------------------------------------------------------------
+__device__ __forceinline__ void pdl_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+__device__ __forceinline__ void pdl_trigger() { asm volatile("griddepcontrol.launch_dependents;" ::: "memory"); }
+
+// Launch with the programmatic-serialisation attribute when `pdl` is set.
+extern bool g_use_pdl;
+template <typename... KArgs, typename... Args>
+inline cudaError_t launch_k(void (*kernel)(KArgs...), dim3 grid, dim3 block, size_t smem, cudaStream_t st,
+                            Args... args) {
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = grid;
+  cfg.blockDim = block;
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = st;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = g_use_pdl ? 1 : 0;
+  return cudaLaunchKernelEx(&cfg, kernel, static_cast<KArgs>(args)...);
+}
+
+// ----------------------------------------------------------------------------
 // Element helpers
 // ----------------------------------------------------------------------------
 typedef __nv_bfloat16 bf16;
@@ -290,7 +319,7 @@ struct PageUpdate {
 };
 
 void launch_router(const ModelDims& md, const StepDev& s, int B, const void* emb, const void* router_w,
-                   const float* router_b, const PageUpdate* upd, int n_upd, cudaStream_t st);
+                   const float* router_b, const PageUpdate* upd, const int* n_upd, cudaStream_t st);
 void launch_plan(const ModelDims& md, const StepDev& s, int B, int target_items, int min_chunk, cudaStream_t st);
 
 void launch_norm_rows(int dtype, const float* H, int ldh, const int* idx, const int* n_dev, int n_host,
