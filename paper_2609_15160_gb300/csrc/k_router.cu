@@ -8,9 +8,9 @@
 //
 // k_plan: one CTA. For every loop r it builds A_r = {b : m_b >= r} in
 // increasing b with a warp ballot plus a block prefix scan, and the work plan
-// of the split-K decode attention over the loop-r caches: the keys per chunk
-// (sized from the device-side cache lengths so that the chunk count is close
-// to a target) and each active token's first work item.
+// of the decode attention over the loop-r caches: the pages of every (token,
+// kv head) item, from the device-side cache lengths, laid out in one flat
+// order (prefix sums), which the attention grid splits evenly.
 #include "tlf_internal.cuh"
 
 namespace tlf {
@@ -139,7 +139,7 @@ __device__ int block_exclusive_scan(int v, int* total) {
   return excl;
 }
 
-__global__ void __launch_bounds__(256) k_plan(ModelDims md, StepDev s, int B, int target_items, int min_chunk) {
+__global__ void __launch_bounds__(256) k_plan(ModelDims md, StepDev s, int B) {
   pdl_wait();
   pdl_trigger();
   const int b = threadIdx.x;
@@ -147,6 +147,8 @@ __global__ void __launch_bounds__(256) k_plan(ModelDims md, StepDev s, int B, in
   const int mb = (b < B) ? s.m[b] : 0;
   const int slot = (b < B) ? s.slots[b] : 0;
   const int maxB = md.max_batch, M = md.M, ps = md.page_size;
+  // attention merge tickets start at zero every step
+  for (int i = b; i < maxB * md.Hkv; i += blockDim.x) s.cnt[i] = 0;
   for (int r = 0; r < M; ++r) {
     const bool active = mb > r;
     // compaction: ballot gives each active lane its rank in the warp, the block scan the warp offsets
@@ -156,24 +158,20 @@ __global__ void __launch_bounds__(256) k_plan(ModelDims md, StepDev s, int B, in
     const int warp_off = block_exclusive_scan((lane == 0) ? __popc(ball) : 0, &n_r);
     const int k = __shfl_sync(0xffffffffu, warp_off, 0) + rank;
     if (active) s.idx[r * maxB + k] = b;
-    // attention plan over the loop-r caches (the token's own new entry included)
+    // attention plan over the loop-r caches (the token's own new entry included): every
+    // (token, kv head) item spans np pages; items are laid out token-major in one flat page order
     const int L = active ? s.len[slot * M + r] + 1 : 0;
-    int tot_keys;
-    (void)block_exclusive_scan(L, &tot_keys);
-    long long want = ((long long)tot_keys * md.Hkv + target_items - 1) / target_items;
-    int ch = (int)(((want + ps - 1) / ps) * ps);
-    if (ch < min_chunk) ch = min_chunk;
-    const int nc = active ? (L + ch - 1) / ch : 0;
-    int items;
-    const int base = block_exclusive_scan(nc * md.Hkv, &items);
+    const int np = (L + ps - 1) / ps;
+    int pages;
+    const int base = block_exclusive_scan(np * md.Hkv, &pages);
     if (active) {
       s.item_base[r * (maxB + 1) + k] = base;
-      s.nch[r * maxB + k] = nc;
+      s.nch[r * maxB + k] = np;
     }
     if (b == 0) {
       s.n[r] = n_r;
-      s.item_base[r * (maxB + 1) + n_r] = items;
-      s.chunk[r] = ch;
+      s.item_base[r * (maxB + 1) + n_r] = pages;
+      s.chunk[r] = ps;
     }
   }
 }
@@ -189,8 +187,8 @@ void launch_router(const ModelDims& md, const StepDev& s, int B, const void* emb
              n_upd);
 }
 
-void launch_plan(const ModelDims& md, const StepDev& s, int B, int target_items, int min_chunk, cudaStream_t st) {
-  launch_k(k_plan, 1, 256, 0, st, md, s, B, target_items, min_chunk);
+void launch_plan(const ModelDims& md, const StepDev& s, int B, cudaStream_t st) {
+  launch_k(k_plan, 1, 256, 0, st, md, s, B);
 }
 
 }  // namespace tlf

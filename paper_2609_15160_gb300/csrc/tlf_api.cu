@@ -97,9 +97,9 @@ struct tlf_ctx {
   int* d_item_base = nullptr;
   int* d_nch = nullptr;
   int* d_chunk = nullptr;
-  float* d_attn_o = nullptr;
-  float* d_attn_ml = nullptr;
-  int attn_grid = 0, attn_target_items = 0, attn_min_chunk = 64;
+  float* d_attn_part = nullptr;
+  int* d_attn_cnt = nullptr;
+  int attn_grid = 0;
   float* d_logits = nullptr;
   uint32_t* d_err = nullptr;
   int* h_m = nullptr;
@@ -423,11 +423,10 @@ static int create_impl(tlf_ctx* ctx, const tlf_weights* w) {
   if ((rc = dev_alloc(ctx, &ctx->d_nch, (size_t)M * B * 4, "nch"))) return rc;
   if ((rc = dev_alloc(ctx, &ctx->d_chunk, (size_t)M * 4, "chunk"))) return rc;
   ctx->attn_grid = attn_decode_grid(md, ctx->num_sms);
-  ctx->attn_target_items = 2 * ctx->attn_grid;
-  const size_t items_max = (size_t)ctx->attn_target_items + (size_t)B * md.Hkv;
-  const int G = md.Hq / md.Hkv;
-  if ((rc = dev_alloc(ctx, &ctx->d_attn_o, items_max * G * md.hd * 4, "attention partials"))) return rc;
-  if ((rc = dev_alloc(ctx, &ctx->d_attn_ml, items_max * G * 2 * 4, "attention partial stats"))) return rc;
+  if ((rc = dev_alloc(ctx, &ctx->d_attn_part, attn_partial_floats(md, ctx->attn_grid) * 4, "attention partials")))
+    return rc;
+  if ((rc = dev_alloc(ctx, &ctx->d_attn_cnt, (size_t)B * md.Hkv * 4, "attention tickets"))) return rc;
+  CK(ctx, cudaMemset(ctx->d_attn_cnt, 0, (size_t)B * md.Hkv * 4));
   if ((rc = dev_alloc(ctx, &ctx->d_logits, (size_t)B * V * 4, "logits"))) return rc;
   if ((rc = dev_alloc(ctx, &ctx->d_err, 16, "error word"))) return rc;
   CK(ctx, cudaMemset(ctx->d_err, 0, 16));
@@ -457,7 +456,7 @@ extern "C" void tlf_destroy(tlf_ctx* ctx) {
     f(ctx->d_pool); f(ctx->d_pos_table); f(ctx->d_page_table); f(ctx->d_len); f(ctx->d_upload);
     f(ctx->d_m); f(ctx->d_margin); f(ctx->d_H); f(ctx->d_X); f(ctx->d_O); f(ctx->d_U); f(ctx->d_Xf);
     f(ctx->d_part); f(ctx->d_Q); f(ctx->d_idx); f(ctx->d_n); f(ctx->d_item_base); f(ctx->d_nch); f(ctx->d_chunk);
-    f(ctx->d_attn_o); f(ctx->d_attn_ml); f(ctx->d_logits); f(ctx->d_err);
+    f(ctx->d_attn_part); f(ctx->d_attn_cnt); f(ctx->d_logits); f(ctx->d_err);
     if (ctx->h_upload) cudaFreeHost(ctx->h_upload);
     if (ctx->h_m) cudaFreeHost(ctx->h_m);
     if (ctx->h_margin) cudaFreeHost(ctx->h_margin);
@@ -605,11 +604,12 @@ static int enqueue_step(tlf_ctx* ctx, int B, bool need_logits, bool prof, cudaSt
   s.pos_table = ctx->d_pos_table;
   s.pool = ctx->d_pool;
   s.err = ctx->d_err;
+  s.cnt = ctx->d_attn_cnt;
   const PageUpdate* d_upd = reinterpret_cast<const PageUpdate*>(ctx->d_upload + 1 + 3 * B);
 
   ctx->last_launches = 0;
   launch_router(md, s, B, ctx->d_emb, ctx->d_router_w, ctx->d_router_b, d_upd, ctx->d_upload, st);
-  launch_plan(md, s, B, ctx->attn_target_items, ctx->attn_min_chunk, st);
+  launch_plan(md, s, B, st);
   ctx->last_launches += 2;
   int ev = 0;
   for (int r = 0; r < M; ++r) {
@@ -627,9 +627,8 @@ static int enqueue_step(tlf_ctx* ctx, int B, bool need_logits, bool prof, cudaSt
       gemm(ctx, ctx->wqkv[j], &ctx->map_X, ctx->d_X, md.d, a, st);
       launch_rope_append(md, s, r, j, ctx->d_part, ctx->s_qkv, ctx->d_Q, ctx->d_inv_freq, st);
       if (prof) cudaEventRecord(ctx->events[ev++], st);
-      launch_attn_decode(md, s, r, j, ctx->d_Q, ctx->d_attn_o, ctx->d_attn_ml, ctx->attn_grid, st);
+      launch_attn_decode(md, s, r, j, ctx->d_Q, ctx->d_attn_part, ctx->d_O, ctx->d_attn_cnt, ctx->attn_grid, st);
       if (prof) cudaEventRecord(ctx->events[ev++], st);
-      launch_attn_combine(md, s, r, ctx->d_attn_o, ctx->d_attn_ml, ctx->d_O, st);
       a = GemmArgs{};
       a.n_dev = n_dev;
       a.max_rows = maxB;
@@ -658,7 +657,7 @@ static int enqueue_step(tlf_ctx* ctx, int B, bool need_logits, bool prof, cudaSt
       a.idx = idx_r;
       a.splits = ctx->s_d;
       gemm(ctx, ctx->wd[j], &ctx->map_U, ctx->d_U, md.ff, a, st);
-      ctx->last_launches += 6;
+      ctx->last_launches += 5;  // 2 norms, RoPE/append, attention, SwiGLU (+4 GEMMs counted in gemm())
     }
   }
   launch_final(md, s, B, ctx->d_final_norm, ctx->d_Xf, st);

@@ -290,7 +290,8 @@ struct StepDev {
   int* n;              // [M] |A_r|
   int* item_base;      // [M][maxB+1]
   int* nch;            // [M][maxB] chunks per token
-  int* chunk;          // [M] keys per chunk
+  int* chunk;          // [M] keys per page
+  int* cnt;            // [maxB * Hkv] attention merge tickets (zeroed by the plan kernel)
   // cache state
   int* len;            // [max_seqs][M] entries per (sequence, loop)
   int* page_table;     // [max_seqs][M][max_pages]
@@ -320,7 +321,7 @@ struct PageUpdate {
 
 void launch_router(const ModelDims& md, const StepDev& s, int B, const void* emb, const void* router_w,
                    const float* router_b, const PageUpdate* upd, const int* n_upd, cudaStream_t st);
-void launch_plan(const ModelDims& md, const StepDev& s, int B, int target_items, int min_chunk, cudaStream_t st);
+void launch_plan(const ModelDims& md, const StepDev& s, int B, cudaStream_t st);
 
 void launch_norm_rows(int dtype, const float* H, int ldh, const int* idx, const int* n_dev, int n_host,
                       int rows_max, const float* gain, int d, float eps, void* X, int ldx, cudaStream_t st);
@@ -332,11 +333,10 @@ int gemm_tc_max_nt();
 
 void launch_rope_append(const ModelDims& md, const StepDev& s, int r, int j, const float* part, int splits,
                         float* Q, const double* inv_freq, cudaStream_t st);
-void launch_attn_decode(const ModelDims& md, const StepDev& s, int r, int j, const float* Q, float* part_o,
-                        float* part_ml, int grid, cudaStream_t st);
-void launch_attn_combine(const ModelDims& md, const StepDev& s, int r, const float* part_o,
-                         const float* part_ml, void* O, cudaStream_t st);
+void launch_attn_decode(const ModelDims& md, const StepDev& s, int r, int j, const float* Q, float* part, void* O,
+                        int* cnt, int grid, cudaStream_t st);
 int attn_decode_grid(const ModelDims& md, int num_sms);
+size_t attn_partial_floats(const ModelDims& md, int grid);
 
 void launch_swiglu(int dtype, const float* part, int splits, int max_rows, const int* n_dev, int ff, void* U,
                    cudaStream_t st);
@@ -348,8 +348,8 @@ void launch_scatter_cache(const ModelDims& md, int slot, int r, int n, const voi
 
 // Kernel-level attention operation (tlf_attn_decode): scratch layout and launch.
 struct AttnOpLayout {
-  size_t m, slots, len, idx, count, item_base, nch, chunk, errw, part_o, part_ml, total;
-  int grid, target_items, items_max;
+  size_t m, slots, len, idx, count, item_base, nch, chunk, errw, cnt, part, total;
+  int grid;
 };
 AttnOpLayout attn_op_layout(const tlf_attn_args* a, int num_sms);
 const char* attn_op_validate(const tlf_attn_args* a);

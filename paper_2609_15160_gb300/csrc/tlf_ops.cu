@@ -31,8 +31,7 @@ AttnOpLayout attn_op_layout(const tlf_attn_args* a, int num_sms) {
   AttnOpLayout L{};
   const int n = a->n, G = a->n_heads / a->n_kv_heads;
   L.grid = 2 * num_sms;
-  L.target_items = 2 * L.grid;
-  L.items_max = L.target_items + n * a->n_kv_heads;
+  const size_t part_floats = ((size_t)n * a->n_kv_heads + L.grid) * G * (a->head_dim + 2);
   size_t o = 0;
   auto take = [&](size_t bytes) { size_t at = o; o = up(o + bytes, 16); return at; };
   L.m = take(4 * (size_t)n);
@@ -44,9 +43,9 @@ AttnOpLayout attn_op_layout(const tlf_attn_args* a, int num_sms) {
   L.nch = take(4 * (size_t)n);
   L.chunk = take(4);
   L.errw = take(4);
+  L.cnt = take(4 * (size_t)n * a->n_kv_heads);
   o = up(o, 256);
-  L.part_o = take(4 * (size_t)L.items_max * G * a->head_dim);
-  L.part_ml = take(4 * (size_t)L.items_max * G * 2);
+  L.part = take(4 * part_floats);
   L.total = up(o, 256);
   return L;
 }
@@ -108,14 +107,13 @@ cudaError_t attn_op_run(const tlf_attn_args* a, uint8_t* scratch, const AttnOpLa
   s.page_table = const_cast<int*>(a->page_table);
   s.pool = const_cast<void*>(a->pool);
   s.err = a->err ? a->err : reinterpret_cast<uint32_t*>(scratch + L.errw);
-  float* part_o = reinterpret_cast<float*>(scratch + L.part_o);
-  float* part_ml = reinterpret_cast<float*>(scratch + L.part_ml);
+  s.cnt = reinterpret_cast<int*>(scratch + L.cnt);
+  float* part = reinterpret_cast<float*>(scratch + L.part);
 
   k_attn_prep<<<(a->n + 127) / 128, 128, 0, st>>>(a->n, a->lens, a->max_pages * a->page_size, s.m,
                                                   const_cast<int*>(s.slots), s.len, s.err);
-  launch_plan(md, s, a->n, L.target_items, 64, st);
-  launch_attn_decode(md, s, 0, a->layer, a->q, part_o, part_ml, L.grid, st);
-  launch_attn_combine(md, s, 0, part_o, part_ml, a->out, st);
+  launch_plan(md, s, a->n, st);
+  launch_attn_decode(md, s, 0, a->layer, a->q, part, a->out, s.cnt, L.grid, st);
   return cudaGetLastError();
 }
 

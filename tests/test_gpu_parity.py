@@ -266,7 +266,7 @@ def test_profile_counters(tlf):
         ctx.set_profiling(True)
         _, loops, _ = ctx.decode_step([1, 2], [5, 6])
         ms, by, nl = ctx.last_step_profile()
-        assert ms > 0 and nl == 2 + m.max_loops * m.n_layers * 10 + 1 + 1
+        assert ms > 0 and nl == 2 + m.max_loops * m.n_layers * 9 + 1 + 1
         want = sum((ctx.cache_len(i, r)) * m.n_layers * 2 * m.n_kv_heads * m.head_dim * 2
                    for i, lp in zip([1, 2], loops) for r in range(1, lp + 1))
         assert abs(by - want) < 1e-6 * want
