@@ -261,6 +261,7 @@ def run_ours(args):
     # --- kernel-level pass: attention kernel time and algorithmic KV bytes ---
     ctx.set_profiling(True)
     att_ms, att_bytes, launches, att_launches = 0.0, 0.0, 0, 0
+    breakdown = {}
     for s in range(args.steps):
         _, lp, _ = ctx.decode_step(ids, toks[2 * n_steps + s], forced=forced, logits=logits_dev, stream=stream)
         ms, by, nl = ctx.last_step_profile()
@@ -268,6 +269,8 @@ def run_ours(args):
         att_bytes += by
         launches += nl
         att_launches += m.n_layers * m.max_loops
+        for kname, kms in ctx.last_step_kernel_times().items():
+            breakdown[kname] = breakdown.get(kname, 0.0) + kms / args.steps
     ctx.set_profiling(False)
 
     times = torch.tensor([total_ms, e2e_ms], dtype=torch.float64, device="cuda")
@@ -302,6 +305,7 @@ def run_ours(args):
             "e2e": {"value": ws * B * args.steps / (e2e_ms * 1e-3), "unit": "tokens/s",
                     "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h},
             "gpu_launches": int(launches),
+            "kernel_ms_per_step_profiled": {k: round(v, 4) for k, v in breakdown.items()},
             "setup_s": setup_s,
         }
         if clk:
@@ -322,7 +326,7 @@ def run_attn_op(args):
 
     T.load_library()
     n, L = args.batch, args.context
-    hq, hkv, hd, J = 16, 8, 128, 2
+    hq, hkv, hd, J = args.hq, args.hkv, args.hd, args.layers
     rng = np.random.default_rng(5)
     need = (L + 63) // 64
     n_pages = n * need + 1
@@ -372,6 +376,10 @@ def main():
     ap.add_argument("--op", default=None, choices=["attn"], help="time one kernel-level operation alone")
     ap.add_argument("--batch", type=int, default=16)
     ap.add_argument("--context", type=int, default=32768)
+    ap.add_argument("--hq", type=int, default=16, help="--op attn: query heads")
+    ap.add_argument("--hkv", type=int, default=8, help="--op attn: kv heads")
+    ap.add_argument("--hd", type=int, default=128, help="--op attn: head dim")
+    ap.add_argument("--layers", type=int, default=2, help="--op attn: layers stored per page")
     ap.add_argument("--gpus", type=int, default=1)
     ap.add_argument("--steps", type=int, default=100)
     ap.add_argument("--warmup", type=int, default=10)

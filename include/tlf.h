@@ -278,6 +278,14 @@ int tlf_set_profiling(tlf_ctx* ctx, int32_t on);
 int tlf_last_step_profile(const tlf_ctx* ctx, float* attn_ms, double* attn_kv_bytes,
                           int32_t* kernel_launches);
 
+/* Per-kernel-class milliseconds of the last decode step run with profiling
+ * on (events between launches, so kernels do not overlap while profiled).
+ * Classes, in order: 0 router, 1 plan (compaction), 2 attention pre-norm,
+ * 3 QKV GEMM, 4 RoPE + append, 5 attention, 6 O GEMM + residual, 7 MLP
+ * pre-norm, 8 gate/up GEMM, 9 SwiGLU, 10 down GEMM + residual, 11 final
+ * norm, 12 LM head. Writes min(n, 13) entries of ms; returns TLF_OK. */
+int tlf_last_step_kernel_times(const tlf_ctx* ctx, float* ms, int32_t n);
+
 #ifdef __cplusplus
 }
 #endif

@@ -46,6 +46,150 @@ constexpr int tc_smem_bytes() {
   return 1024 /*align slack*/ + TC_STAGES * (TC_BM * TC_BK * 2 + NT * TC_BK * 2) + 256 /*barriers, tmem slot*/;
 }
 
+// Second half of a cluster epilogue. Every CTA of the cluster has staged its
+// fp32 partial tile [128 features][NT + 1] at `red`; this CTA sums the partners'
+// tiles over its share of the token columns through distributed shared memory
+// and finishes them according to the mode.
+constexpr int CL_MAX = 8;  // largest cluster (split-K factor) of the cluster epilogues
+
+// Sums over the cluster of the staged values at feature f, columns c..c+3
+// (columns >= c1 give 0). All partner loads of the four columns are issued
+// before any is used.
+__device__ __forceinline__ void cluster_sum4(const uint32_t* pb, int S, int f, int c, int c1, float out[4]) {
+  float v[CL_MAX][4];
+#pragma unroll
+  for (int p = 0; p < CL_MAX; ++p)
+#pragma unroll
+    for (int q = 0; q < 4; ++q)
+      v[p][q] = (p < S && c + q < c1) ? dsmem_ld_f32(pb[p] + 4u * (uint32_t)((c + q) * 128 + f)) : 0.f;
+#pragma unroll
+  for (int q = 0; q < 4; ++q) {
+    float s = 0.f;
+#pragma unroll
+    for (int p = 0; p < CL_MAX; ++p) s += v[p][q];
+    out[q] = s;
+  }
+}
+
+template <int NT>
+__device__ void cluster_epilogue(const GemmArgs& a, float* red, int* colinfo, int m0, int n) {
+  const int S = a.splits;
+  const int rank = (int)cluster_ctarank();
+  const int per = (n + S - 1) / S;
+  const int c0 = rank * per, c1 = min(n, c0 + per);
+  const int tid = threadIdx.x;
+  uint32_t pb[CL_MAX];
+  const uint32_t base = smem_u32(red);
+#pragma unroll
+  for (int p = 0; p < CL_MAX; ++p) pb[p] = (p < S) ? dsmem_map(base, (uint32_t)p) : 0u;
+
+  if (a.epi == EPI_CL_RESID) {
+    const int col = m0 + tid;
+    if (col < a.N)
+      for (int c = c0; c < c1; c += 4) {
+        float sm[4];
+        cluster_sum4(pb, S, tid, c, c1, sm);
+#pragma unroll
+        for (int q = 0; q < 4; ++q)
+          if (c + q < c1) {
+            const int row = a.idx ? a.idx[c + q] : c + q;
+            atomicAdd(a.resid + (size_t)row * a.ldr + col, sm[q]);  // the only writer of this element
+          }
+      }
+    return;
+  }
+  if (a.epi == EPI_CL_SWIGLU) {
+    const int gf = (m0 >> 1) + tid;  // 64 gate rows then 64 up rows per 128-row tile
+    if (tid < 64 && gf < a.md.ff)
+      for (int c = c0; c < c1; c += 4) {
+        float g[4], u[4];
+        cluster_sum4(pb, S, tid, c, c1, g);
+        cluster_sum4(pb, S, tid + 64, c, c1, u);
+#pragma unroll
+        for (int q = 0; q < 4; ++q)
+          if (c + q < c1)
+            reinterpret_cast<bf16*>(a.U)[(size_t)(c + q) * a.md.ff + gf] =
+                __float2bfloat16_rn(g[q] / (1.f + expf(-g[q])) * u[q]);
+      }
+    return;
+  }
+  // EPI_CL_QKV: column c is token k = c of A_r
+  const ModelDims& md = a.md;
+  const StepDev& s = a.s;
+  const int ps = md.page_size, hd = md.hd, half = hd / 2;
+  int* ci_pos = colinfo;
+  int* ci_page = colinfo + NT;
+  int* ci_off = colinfo + 2 * NT;
+  for (int t = tid; t < c1 - c0; t += blockDim.x) {
+    const int c = c0 + t;
+    const int b = s.idx[a.r * md.max_batch + c];
+    const int slot = s.slots[b];
+    const int L = s.len[slot * md.M + a.r];
+    int page = s.page_table[((size_t)slot * md.M + a.r) * md.max_pages + L / ps];
+    if (page < 0 || page >= md.n_pages) {
+      atomicOr(s.err, DEVERR_INDEX);
+      page = -1;
+    }
+    ci_pos[t] = s.len[slot * md.M];  // every token runs loop 1: its length is the token count
+    ci_page[t] = page;
+    ci_off[t] = L % ps;
+    if (a.j == 0 && page >= 0) s.pos_table[(size_t)page * ps + L % ps] = ci_pos[t];
+  }
+  __syncthreads();
+  const int gfeat = m0 + tid;
+  if (gfeat >= md.qkv_dim) return;
+  const double two_pi = 6.283185307179586476925286766559;
+  bf16* pool = reinterpret_cast<bf16*>(s.pool);
+  if (gfeat < md.q_dim + md.kv_dim) {
+    const bool is_q = gfeat < md.q_dim;
+    const int fr = is_q ? gfeat : gfeat - md.q_dim;
+    const int h = fr / hd, i = fr % hd;
+    if (i >= half) return;  // the lower lane of the rotary pair handles both
+    const double freq = a.inv_freq[i];
+    for (int c = c0; c < c1; c += 4) {
+      float x0[4], x1[4];
+      cluster_sum4(pb, S, tid, c, c1, x0);
+      cluster_sum4(pb, S, tid + half, c, c1, x1);
+#pragma unroll
+      for (int q = 0; q < 4; ++q) {
+        const int cc = c + q;
+        if (cc >= c1) break;
+        double ang = (double)ci_pos[cc - c0] * freq;
+        ang -= two_pi * rint(ang / two_pi);
+        float sn, cs;
+        sincosf((float)ang, &sn, &cs);
+        const float r0 = x0[q] * cs - x1[q] * sn, r1 = x0[q] * sn + x1[q] * cs;
+        if (is_q) {
+          float* qo = a.Q + ((size_t)cc * md.Hq + h) * hd;
+          qo[i] = r0;
+          qo[i + half] = r1;
+        } else if (ci_page[cc - c0] >= 0) {
+          bf16* kp = pool + (size_t)ci_page[cc - c0] * md.page_elems +
+                     ((size_t)(a.j * 2 + 0) * md.Hkv + h) * ps * hd + (size_t)ci_off[cc - c0] * hd;
+          kp[i] = __float2bfloat16_rn(r0);
+          kp[i + half] = __float2bfloat16_rn(r1);
+        }
+      }
+    }
+  } else {
+    const int fr = gfeat - md.q_dim - md.kv_dim;
+    const int h = fr / hd, i = fr % hd;
+    for (int c = c0; c < c1; c += 4) {
+      float x[4];
+      cluster_sum4(pb, S, tid, c, c1, x);
+#pragma unroll
+      for (int q = 0; q < 4; ++q) {
+        const int cc = c + q;
+        if (cc < c1 && ci_page[cc - c0] >= 0) {
+          bf16* vp = pool + (size_t)ci_page[cc - c0] * md.page_elems +
+                     ((size_t)(a.j * 2 + 1) * md.Hkv + h) * ps * hd + (size_t)ci_off[cc - c0] * hd;
+          vp[i] = __float2bfloat16_rn(x[q]);
+        }
+      }
+    }
+  }
+}
+
 template <int NT>
 __global__ void __launch_bounds__(128) k_gemm_tc(const __grid_constant__ CUtensorMap mapW,
                                                  const __grid_constant__ CUtensorMap mapX, GemmArgs a) {
@@ -150,6 +294,33 @@ __global__ void __launch_bounds__(128) k_gemm_tc(const __grid_constant__ CUtenso
   if (nk > 0) ok = mbar_wait(done, 0, a.err);
   ok = __all_sync(0xffffffffu, ok);  // tcgen05.ld is warp-collective
   tc_fence_after();
+  if (a.epi >= EPI_CL_RESID) {
+    // Stage the partial tile in shared memory (the operand ring is free now),
+    // then reduce across the cluster. Every CTA reaches both cluster barriers.
+    // tile layout [column][128 features]: a warp's partner reads are 128 contiguous bytes
+    float* red = reinterpret_cast<float*>(smem);
+    int* colinfo = reinterpret_cast<int*>(red + 128 * NT);
+    const int f = warp * 32 + lane;
+    for (int c0 = 0; c0 < ncols; c0 += 16) {
+      float v[16];
+      if (ok && nk > 0) {
+        tmem_ld_16(tmem + ((uint32_t)(warp * 32) << 16) + (uint32_t)c0, v);
+      } else {
+#pragma unroll
+        for (int i = 0; i < 16; ++i) v[i] = 0.f;
+      }
+#pragma unroll
+      for (int i = 0; i < 16; ++i) red[(c0 + i) * 128 + f] = v[i];
+    }
+    tc_fence_before();
+    __syncthreads();
+    if (warp == 0) tmem_dealloc(tmem, TMEM_COLS);
+    cluster_sync_all();  // every partner's tile is staged
+    cluster_epilogue<NT>(a, red, colinfo, m0, n);
+    __syncwarp();
+    cluster_sync_all();  // partners have finished reading this CTA's tile
+    return;
+  }
   if (ok) {
     const int col = m0 + warp * 32 + lane;
     for (int c0 = 0; c0 < ncols; c0 += 16) {
@@ -183,7 +354,31 @@ static void launch_tc_nt(const CUtensorMap* mapW, const CUtensorMap* mapX, const
     attr_set = true;
   }
   dim3 grid((a.N + TC_BM - 1) / TC_BM, a.splits);
-  launch_k(k_gemm_tc<NT>, grid, 128, smem, st, *mapW, *mapX, a);
+  if (a.epi < EPI_CL_RESID) {
+    launch_k(k_gemm_tc<NT>, grid, 128, smem, st, *mapW, *mapX, a);
+    return;
+  }
+  // cluster epilogue: the splits of one tile form a (1, splits, 1) cluster
+  static bool nonportable = false;
+  if (a.splits > 8 && !nonportable) {
+    cudaFuncSetAttribute(k_gemm_tc<NT>, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
+    nonportable = true;
+  }
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = grid;
+  cfg.blockDim = dim3(128);
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = st;
+  cudaLaunchAttribute attr[2];
+  attr[0].id = cudaLaunchAttributeClusterDimension;
+  attr[0].val.clusterDim.x = 1;
+  attr[0].val.clusterDim.y = a.splits;
+  attr[0].val.clusterDim.z = 1;
+  attr[1].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[1].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = g_use_pdl ? 2 : 1;
+  cudaLaunchKernelEx(&cfg, k_gemm_tc<NT>, *mapW, *mapX, a);
 }
 
 void launch_gemm_tc(const CUtensorMap* mapW, const CUtensorMap* mapX, int nt_max, const GemmArgs& a,

@@ -113,7 +113,8 @@ struct tlf_ctx {
   double last_attn_bytes = 0.0;
   int last_launches = 0;
   std::vector<cudaEvent_t> events;
-  int n_events = 0;
+  std::vector<int> ev_class;  // kernel class closed by each profiling event
+  float class_ms[13] = {};
   int last_batch = 0;
 
   // CUDA graphs of the step
@@ -359,7 +360,25 @@ static int create_impl(tlf_ctx* ctx, const tlf_weights* w) {
     if ((rc = make_mat(ctx, &ctx->wo[j], {o}, {d}, md.q_dim, "wo"))) return rc;
     const uint8_t* gt = (const uint8_t*)w->w_gate + (size_t)j * ff * d * eb;
     const uint8_t* up = (const uint8_t*)w->w_up + (size_t)j * ff * d * eb;
-    if ((rc = make_mat(ctx, &ctx->wgu[j], {gt, up}, {ff, ff}, d, "w_gate_up"))) return rc;
+    if (ctx->use_tc) {
+      // 128-row tiles of 64 gate rows then the 64 matching up rows (zero rows past ff), so the
+      // GEMM epilogue sees both halves of SwiGLU in one tile
+      const int tiles = (ff + 63) / 64;
+      const size_t rb = (size_t)d * eb;
+      std::vector<uint8_t> zero(rb * 64, 0);
+      std::vector<const uint8_t*> parts;
+      std::vector<int> rows;
+      for (int t = 0; t < tiles; ++t) {
+        const int cnt = std::min(64, ff - 64 * t);
+        parts.push_back(gt + (size_t)64 * t * rb); rows.push_back(cnt);
+        if (cnt < 64) { parts.push_back(zero.data()); rows.push_back(64 - cnt); }
+        parts.push_back(up + (size_t)64 * t * rb); rows.push_back(cnt);
+        if (cnt < 64) { parts.push_back(zero.data()); rows.push_back(64 - cnt); }
+      }
+      if ((rc = make_mat(ctx, &ctx->wgu[j], parts, rows, d, "w_gate_up"))) return rc;
+    } else if ((rc = make_mat(ctx, &ctx->wgu[j], {gt, up}, {ff, ff}, d, "w_gate_up"))) {
+      return rc;
+    }
     const uint8_t* dn = (const uint8_t*)w->w_down + (size_t)j * d * ff * eb;
     if ((rc = make_mat(ctx, &ctx->wd[j], {dn}, {d}, ff, "w_down"))) return rc;
   }
@@ -401,12 +420,13 @@ static int create_impl(tlf_ctx* ctx, const tlf_weights* w) {
   }
   // split-K factors: enough CTAs to cover the SMs (2 per SM when the tile is small)
   if (ctx->use_tc) {
+    // the splits of a tile form one thread-block cluster (at most 8 CTAs, the portable size)
     const int per_sm = ctx->nt_max <= 64 ? 2 : 1;
     const int target = per_sm * ctx->num_sms;
-    ctx->s_qkv = choose_splits((md.qkv_dim + 127) / 128, (d + 63) / 64, target, ctx->split_cap);
-    ctx->s_o = choose_splits((d + 127) / 128, (md.q_dim + 63) / 64, target, 32);
-    ctx->s_gu = choose_splits((2 * ff + 127) / 128, (d + 63) / 64, target, ctx->split_cap);
-    ctx->s_d = choose_splits((d + 127) / 128, (ff + 63) / 64, target, 32);
+    ctx->s_qkv = choose_splits((md.qkv_dim + 127) / 128, (d + 63) / 64, target, 8);
+    ctx->s_o = choose_splits((d + 127) / 128, (md.q_dim + 63) / 64, target, 8);
+    ctx->s_gu = choose_splits(ctx->wgu[0].N / 128, (d + 63) / 64, target, 8);
+    ctx->s_d = choose_splits((d + 127) / 128, (ff + 63) / 64, target, 8);
   } else {
     const int target = 2 * ctx->num_sms;
     ctx->s_qkv = choose_splits((md.qkv_dim + 63) / 64, (d + 31) / 32, target, ctx->split_cap);
@@ -438,7 +458,7 @@ static int create_impl(tlf_ctx* ctx, const tlf_weights* w) {
     const char* e = getenv("TLF_NO_GRAPH");
     ctx->use_graphs = !(e && e[0] == '1');
   }
-  ctx->events.resize(2 * M * J + 2);
+  ctx->events.resize(4 + 9 * (size_t)M * J + 2);
   for (auto& e : ctx->events) CK(ctx, cudaEventCreate(&e));
   CK(ctx, cudaDeviceSynchronize());
   return TLF_OK;
@@ -608,61 +628,101 @@ static int enqueue_step(tlf_ctx* ctx, int B, bool need_logits, bool prof, cudaSt
   const PageUpdate* d_upd = reinterpret_cast<const PageUpdate*>(ctx->d_upload + 1 + 3 * B);
 
   ctx->last_launches = 0;
-  launch_router(md, s, B, ctx->d_emb, ctx->d_router_w, ctx->d_router_b, d_upd, ctx->d_upload, st);
-  launch_plan(md, s, B, st);
-  ctx->last_launches += 2;
   int ev = 0;
+  ctx->ev_class.clear();
+  // profiling: an event after every launch, tagged with the kernel class it closes
+  auto mark = [&](int cls) {
+    if (!prof) return;
+    cudaEventRecord(ctx->events[ev++], st);
+    if (cls >= 0) ctx->ev_class.push_back(cls);
+  };
+  mark(-1);
+  launch_router(md, s, B, ctx->d_emb, ctx->d_router_w, ctx->d_router_b, d_upd, ctx->d_upload, st);
+  mark(0);
+  launch_plan(md, s, B, st);
+  mark(1);
+  ctx->last_launches += 2;
   for (int r = 0; r < M; ++r) {
     const int* n_dev = ctx->d_n + r;
     const int* idx_r = ctx->d_idx + (size_t)r * maxB;
     for (int j = 0; j < J; ++j) {
       launch_norm_rows(md.dtype, ctx->d_H, md.d, idx_r, n_dev, 0, maxB, ctx->d_attn_norm + (size_t)j * md.d, md.d,
                        md.eps, ctx->d_X, md.d, st);
+      mark(2);
       GemmArgs a{};
       a.n_dev = n_dev;
       a.max_rows = maxB;
-      a.epi = EPI_PARTIAL;
-      a.out = ctx->d_part;
       a.splits = ctx->s_qkv;
-      gemm(ctx, ctx->wqkv[j], &ctx->map_X, ctx->d_X, md.d, a, st);
-      launch_rope_append(md, s, r, j, ctx->d_part, ctx->s_qkv, ctx->d_Q, ctx->d_inv_freq, st);
-      if (prof) cudaEventRecord(ctx->events[ev++], st);
+      if (ctx->use_tc) {
+        // split-K reduction, RoPE and the K/V append run in the GEMM's cluster epilogue
+        a.epi = EPI_CL_QKV;
+        a.md = md;
+        a.s = s;
+        a.r = r;
+        a.j = j;
+        a.inv_freq = ctx->d_inv_freq;
+        a.Q = ctx->d_Q;
+        gemm(ctx, ctx->wqkv[j], &ctx->map_X, ctx->d_X, md.d, a, st);
+        mark(3);
+      } else {
+        a.epi = EPI_PARTIAL;
+        a.out = ctx->d_part;
+        gemm(ctx, ctx->wqkv[j], &ctx->map_X, ctx->d_X, md.d, a, st);
+        mark(3);
+        launch_rope_append(md, s, r, j, ctx->d_part, ctx->s_qkv, ctx->d_Q, ctx->d_inv_freq, st);
+        ++ctx->last_launches;
+        mark(4);
+      }
       launch_attn_decode(md, s, r, j, ctx->d_Q, ctx->d_attn_part, ctx->d_O, ctx->d_attn_cnt, ctx->attn_grid, st);
-      if (prof) cudaEventRecord(ctx->events[ev++], st);
+      mark(5);
       a = GemmArgs{};
       a.n_dev = n_dev;
       a.max_rows = maxB;
-      a.epi = EPI_RESID;
+      a.epi = ctx->use_tc ? EPI_CL_RESID : EPI_RESID;
       a.resid = ctx->d_H;
       a.ldr = md.d;
       a.idx = idx_r;
       a.splits = ctx->s_o;
       gemm(ctx, ctx->wo[j], &ctx->map_O, ctx->d_O, md.q_dim, a, st);
+      mark(6);
       launch_norm_rows(md.dtype, ctx->d_H, md.d, idx_r, n_dev, 0, maxB, ctx->d_mlp_norm + (size_t)j * md.d, md.d,
                        md.eps, ctx->d_X, md.d, st);
+      mark(7);
       a = GemmArgs{};
       a.n_dev = n_dev;
       a.max_rows = maxB;
-      a.epi = EPI_PARTIAL;
-      a.out = ctx->d_part;
       a.splits = ctx->s_gu;
-      gemm(ctx, ctx->wgu[j], &ctx->map_X, ctx->d_X, md.d, a, st);
-      launch_swiglu(md.dtype, ctx->d_part, ctx->s_gu, maxB, n_dev, md.ff, ctx->d_U, st);
+      if (ctx->use_tc) {
+        a.epi = EPI_CL_SWIGLU;  // SwiGLU in the cluster epilogue
+        a.md = md;
+        a.U = ctx->d_U;
+        gemm(ctx, ctx->wgu[j], &ctx->map_X, ctx->d_X, md.d, a, st);
+        mark(8);
+      } else {
+        a.epi = EPI_PARTIAL;
+        a.out = ctx->d_part;
+        gemm(ctx, ctx->wgu[j], &ctx->map_X, ctx->d_X, md.d, a, st);
+        mark(8);
+        launch_swiglu(md.dtype, ctx->d_part, ctx->s_gu, maxB, n_dev, md.ff, ctx->d_U, st);
+        ++ctx->last_launches;
+        mark(9);
+      }
       a = GemmArgs{};
       a.n_dev = n_dev;
       a.max_rows = maxB;
-      a.epi = EPI_RESID;
+      a.epi = ctx->use_tc ? EPI_CL_RESID : EPI_RESID;
       a.resid = ctx->d_H;
       a.ldr = md.d;
       a.idx = idx_r;
       a.splits = ctx->s_d;
       gemm(ctx, ctx->wd[j], &ctx->map_U, ctx->d_U, md.ff, a, st);
-      ctx->last_launches += 5;  // 2 norms, RoPE/append, attention, SwiGLU (+4 GEMMs counted in gemm())
+      mark(10);
+      ctx->last_launches += 3;  // 2 norms and the attention (GEMMs counted in gemm())
     }
   }
   launch_final(md, s, B, ctx->d_final_norm, ctx->d_Xf, st);
+  mark(11);
   ++ctx->last_launches;
-  ctx->n_events = ev;
   if (need_logits) {
     GemmArgs a{};
     a.n_host = B;
@@ -672,6 +732,7 @@ static int enqueue_step(tlf_ctx* ctx, int B, bool need_logits, bool prof, cudaSt
     a.ldo = md.V;
     a.splits = 1;
     gemm(ctx, ctx->emb_mat, &ctx->map_Xf, ctx->d_Xf, md.d, a, st);
+    mark(12);
   }
   CK(ctx, cudaGetLastError());
   CK(ctx, cudaMemcpyAsync(ctx->h_m, ctx->d_m, (size_t)B * 4, cudaMemcpyDeviceToHost, st));
@@ -738,13 +799,13 @@ static int run_step(tlf_ctx* ctx, int B, const int* slots, const int* tokens, co
     return fail(ctx, TLF_ERR_DEVICE, "device error word 0x%x (1 = bounded wait expired, 2 = bad index)", e);
   }
   if (prof) {
-    float tot = 0.f;
-    for (int i = 0; i + 1 < ctx->n_events; i += 2) {
+    for (float& c : ctx->class_ms) c = 0.f;
+    for (size_t i = 0; i < ctx->ev_class.size(); ++i) {
       float ms = 0.f;
       cudaEventElapsedTime(&ms, ctx->events[i], ctx->events[i + 1]);
-      tot += ms;
+      ctx->class_ms[ctx->ev_class[i]] += ms;
     }
-    ctx->last_attn_ms = tot;
+    ctx->last_attn_ms = ctx->class_ms[5];
     // KV bytes visited: for every row b and loop r < m_b, (len + 1) entries x J layers x K,V
     double bytes = 0.0;
     for (int b = 0; b < B; ++b)
@@ -1050,5 +1111,11 @@ extern "C" int tlf_last_step_profile(const tlf_ctx* ctx, float* attn_ms, double*
   if (attn_ms) *attn_ms = ctx->last_attn_ms;
   if (attn_kv_bytes) *attn_kv_bytes = ctx->last_attn_bytes;
   if (kernel_launches) *kernel_launches = ctx->last_launches;
+  return TLF_OK;
+}
+
+extern "C" int tlf_last_step_kernel_times(const tlf_ctx* ctx, float* ms, int32_t n) {
+  if (!ctx || !ms || n < 0) return TLF_ERR_INVALID_ARG;
+  for (int i = 0; i < n && i < 13; ++i) ms[i] = ctx->class_ms[i];
   return TLF_OK;
 }

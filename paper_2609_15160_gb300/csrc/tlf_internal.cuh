@@ -239,6 +239,34 @@ __host__ __device__ constexpr uint32_t idesc_bf16_f32(int M, int N) {
 }
 
 // ----------------------------------------------------------------------------
+// Thread-block clusters: rank, distributed shared memory, cluster barrier.
+// Every CTA of a cluster is resident at the same time, so the barrier always
+// completes once each CTA of the cluster reaches it (no CTA returns early).
+// ----------------------------------------------------------------------------
+__device__ __forceinline__ uint32_t cluster_ctarank() {
+  uint32_t r;
+  asm volatile("mov.u32 %0, %%cluster_ctarank;" : "=r"(r));
+  return r;
+}
+// Address of the same shared-memory location in CTA `rank` of the cluster.
+__device__ __forceinline__ uint32_t dsmem_map(uint32_t saddr, uint32_t rank) {
+  uint32_t r;
+  asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(r) : "r"(saddr), "r"(rank));
+  return r;
+}
+// Not volatile: the address comes from dsmem_map (volatile, issued after the
+// cluster barrier), so these loads cannot move above the barrier but can be
+// batched freely.
+__device__ __forceinline__ float dsmem_ld_f32(uint32_t addr) {
+  float v;
+  asm("ld.shared::cluster.f32 %0, [%1];" : "=f"(v) : "r"(addr));
+  return v;
+}
+__device__ __forceinline__ void cluster_sync_all() {
+  asm volatile("barrier.cluster.arrive.release.aligned;\n\tbarrier.cluster.wait.acquire.aligned;" ::: "memory");
+}
+
+// ----------------------------------------------------------------------------
 // Warp / block reductions and scans
 // ----------------------------------------------------------------------------
 __device__ __forceinline__ float warp_sum(float v) {
@@ -256,25 +284,16 @@ __device__ __forceinline__ float warp_max(float v) {
 // Kernel argument blocks
 // ----------------------------------------------------------------------------
 enum GemmEpilogue : int {
-  EPI_PARTIAL = 0,  // out[s][row][col] = acc (split-K partial sums, float32)
-  EPI_RESID = 1,    // atomicAdd(resid[idx[row]][col], acc) (residual add + scatter, Eq. 7)
-  EPI_STORE = 2,    // out[row][col] = acc (float32; single split)
-};
-
-struct GemmArgs {
-  int N;             // output features (rows of W)
-  int K;             // reduction length
-  int splits;        // split-K factor (gridDim.y)
-  const int* n_dev;  // token rows n (device scalar), or NULL to use n_host
-  int n_host;
-  int epi;           // GemmEpilogue
-  float* out;        // EPI_PARTIAL: [splits][max_rows][N]; EPI_STORE: [rows][ldo]
-  int ldo;
-  int max_rows;
-  float* resid;      // EPI_RESID: [*][ldr]
-  int ldr;
-  const int* idx;    // EPI_RESID row map (NULL = identity)
-  uint32_t* err;
+  EPI_PARTIAL = 0,    // out[s][row][col] = acc (split-K partial sums, float32)
+  EPI_RESID = 1,      // atomicAdd(resid[idx[row]][col], acc) (residual add + scatter, Eq. 7)
+  EPI_STORE = 2,      // out[row][col] = acc (float32; single split)
+  // Cluster epilogues: the split-K CTAs of a tile form one cluster and sum their
+  // partial tiles through distributed shared memory, then:
+  EPI_CL_RESID = 3,   // resid[idx[row]][col] += sum (one writer per element; Eq. 7)
+  EPI_CL_QKV = 4,     // RoPE on q and k at the original position, q -> Q, k and v appended to
+                      // the loop-r page of the token's sequence (Eq. 9, 11)
+  EPI_CL_SWIGLU = 5,  // U[row][64*tile + f] = silu(gate_f) * up_f; each 128-row weight tile holds
+                      // 64 gate rows then the 64 matching up rows
 };
 
 struct StepDev {
@@ -309,6 +328,29 @@ struct ModelDims {
   float eps, rope_base, threshold;
   int exit_rule;
   int dtype;             // 0 f32, 1 bf16
+};
+
+struct GemmArgs {
+  int N;             // output features (rows of W)
+  int K;             // reduction length
+  int splits;        // split-K factor (gridDim.y; the cluster size for EPI_CL_*)
+  const int* n_dev;  // token rows n (device scalar), or NULL to use n_host
+  int n_host;
+  int epi;           // GemmEpilogue
+  float* out;        // EPI_PARTIAL: [splits][max_rows][N]; EPI_STORE: [rows][ldo]
+  int ldo;
+  int max_rows;
+  float* resid;      // EPI_RESID / EPI_CL_RESID: [*][ldr]
+  int ldr;
+  const int* idx;    // residual row map (NULL = identity)
+  uint32_t* err;
+  // EPI_CL_QKV / EPI_CL_SWIGLU
+  ModelDims md;
+  StepDev s;
+  int r, j;
+  const double* inv_freq;  // [hd/2] rotary frequencies
+  float* Q;                // [max_rows][Hq][hd]
+  void* U;                 // [max_rows][ff] bf16
 };
 
 // ----------------------------------------------------------------------------

@@ -20,6 +20,8 @@ TLF_OK = 0
 ERRORS = {-1: "INVALID_ARG", -2: "UNKNOWN_SEQ", -3: "DUPLICATE_SEQ", -4: "OUT_OF_PAGES", -5: "SEQ_TOO_LONG",
           -6: "CUDA", -7: "BAD_WEIGHTS", -8: "DEVICE", -9: "NO_DEVICE", -10: "CAPACITY"}
 CODES = {v: k for k, v in ERRORS.items()}
+KERNEL_CLASSES = ("router", "plan", "attn_norm", "qkv_gemm", "rope_append", "attention", "o_gemm", "mlp_norm",
+                  "gate_up_gemm", "swiglu", "down_gemm", "final_norm", "lm_head")
 DTYPE = {"f32": 0, "bf16": 1}
 EXIT = {"argmax": 0, "survival": 1}
 GEMM = {"auto": 0, "simt": 1}
@@ -74,6 +76,7 @@ _SIGS = {
     "tlf_last_active_sets": (C.c_int, [_P, _I32P, _I32P]),
     "tlf_set_profiling": (C.c_int, [_P, C.c_int32]),
     "tlf_last_step_profile": (C.c_int, [_P, _F32P, C.POINTER(C.c_double), _I32P]),
+    "tlf_last_step_kernel_times": (C.c_int, [_P, _F32P, C.c_int32]),
     "tlf_attn_decode_scratch_bytes": (C.c_size_t, [C.POINTER(TlfAttnArgs)]),
     "tlf_attn_decode": (C.c_int, [C.POINTER(TlfAttnArgs), _P, C.c_size_t, _P]),
     "tlf_attn_decode_static": (C.c_int, [C.POINTER(TlfAttnArgs), _P]),
@@ -338,3 +341,9 @@ class Context:
         ms, by, nl = C.c_float(), C.c_double(), C.c_int32()
         _check(load_library().tlf_last_step_profile(self.handle, C.byref(ms), C.byref(by), C.byref(nl)), self.handle)
         return ms.value, by.value, nl.value
+
+    def last_step_kernel_times(self) -> Dict[str, float]:
+        """Milliseconds per kernel class of the last profiled step."""
+        ms = np.zeros(len(KERNEL_CLASSES), dtype=np.float32)
+        _check(load_library().tlf_last_step_kernel_times(self.handle, _ptr(ms, C.c_float), len(ms)), self.handle)
+        return dict(zip(KERNEL_CLASSES, ms.tolist()))
