@@ -177,14 +177,17 @@ def setup_workload(T, wl, rank: int, gemm_impl="auto", prefill="auto", extra_tok
     use_snapshot = prefill == "snapshot" or (prefill == "auto" and max(lengths) > 4096)
     ids = [rank * 100000 + b for b in range(B)]
     if use_snapshot:
+        # uniform lengths: two distinct host snapshots (values uploaded); ragged lengths: one
+        # snapshot per sequence with only positions, values filled on the device
+        host_values = wl.prompt_len[0] == wl.prompt_len[1]
         distinct = {}
         snaps = []
         for b, L in enumerate(lengths):
-            key = (L, b % 2) if wl.prompt_len[0] == wl.prompt_len[1] else (L, 0)
+            key = (L, b % 2) if host_values else (L, b)
             if key not in distinct:
-                distinct[key] = synth.make_cache_snapshot(m, L, seed=1000 * rank + len(distinct),
-                                                          depths=None if wl.forced_loops is None else
-                                                          np.full(L, wl.forced_loops, np.int32))
+                depths = None if wl.forced_loops is None else np.full(L, wl.forced_loops, np.int32)
+                make = synth.make_cache_snapshot if host_values else synth.make_cache_positions
+                distinct[key] = make(m, L, seed=1000 * rank + len(distinct), depths=depths)
             snaps.append(distinct[key])
         pages = sum(sum((len(p) + 63) // 64 for p in s["positions"]) for s in snaps) + B * m.max_loops * (
             steps_cap // 64 + 2)
@@ -199,7 +202,13 @@ def setup_workload(T, wl, rank: int, gemm_impl="auto", prefill="auto", extra_tok
     else:
         forced = None if wl.forced_loops is None else [np.full(len(p), wl.forced_loops, np.int32) for p in prompts]
         ctx.prefill(ids, prompts, forced=forced, logits=False)
-    return ctx, ids, "restored synthetic snapshot" if snaps is not None else "prefill through the library"
+    if snaps is None:
+        how = "prefill through the library"
+    elif "k" in snaps[0]:
+        how = "restored synthetic snapshot (host values)"
+    else:
+        how = "restored synthetic snapshot (values filled on the device)"
+    return ctx, ids, how
 
 
 def run_ours(args):
@@ -214,6 +223,8 @@ def run_ours(args):
         dist.init_process_group("nccl")
     T.load_library()
     wl = synth.get_config(args.config)
+    if args.decode_batch:
+        wl = wl.with_batch(args.decode_batch)
     m = wl.model
     B = wl.batch
     t0 = time.time()
@@ -277,6 +288,17 @@ def run_ours(args):
     if ws > 1:
         torch.distributed.all_reduce(times, op=torch.distributed.ReduceOp.MAX)
     total_ms, e2e_ms = times.tolist()
+    # algorithmic HBM bytes of the timed steps: the weights of every loop that had an active
+    # token (read once per loop), the LM head, and the K/V every active token reads and writes
+    eb = 2 if m.dtype == "bf16" else 4
+    w_loop = m.n_layers * m.layer_params() * eb
+    kv_entry = m.n_layers * 2 * m.n_kv_heads * m.head_dim * eb
+    step_bytes = []
+    for lp in loops_seen:
+        loops_run = int(lp.max())
+        step_bytes.append(loops_run * w_loop + m.vocab * m.d_model * eb + int(lp.sum()) * kv_entry)
+    kv_read_per_step = att_bytes / args.steps
+    alg_bytes = float(np.mean(step_bytes)) + kv_read_per_step
     loops_seen = np.concatenate(loops_seen)
     if rank == 0:
         peak, peak_kind = _measured_peaks()
@@ -295,6 +317,10 @@ def run_ours(args):
                        "l2": "inputs larger than L2 (KV cache and weights stream from HBM every step)",
                        "parallelism": f"replicas x{ws} (independent sequences per GPU)"},
             "mean_loops": float(loops_seen.mean()),
+            "step_roofline": {"bound": "hbm", "algorithmic_bytes_per_step": alg_bytes,
+                              "floor_ms": alg_bytes / (peak * 1e9) * 1e3,
+                              "frac": (alg_bytes / (peak * 1e9) * 1e3) / (total_ms / args.steps),
+                              "peak_gbs": peak, "peak_kind": peak_kind},
             "attention_gbs": att_gbs,
             "roofline": {"bound": "hbm", "kernel": "k_attn_decode (recursion-wise split-K attention)",
                          "achieved": att_gbs, "peak": peak, "unit": "GB/s",
@@ -387,6 +413,7 @@ def main():
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--prefill", default="auto", choices=["auto", "snapshot", "real"])
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--decode-batch", type=int, default=0, help="override the workload's batch (C5 sweep)")
     args = ap.parse_args()
     if args.warmup < 3:
         args.warmup = 3

@@ -187,6 +187,10 @@ int tlf_release(tlf_ctx* ctx, uint64_t seq_id);
  * nest, Eq. 4-5). k and v are host arrays in the config dtype laid out
  * [sum lens][J][Hkv][hd] in the same loop order, already rotated (RoPE at
  * their positions). The next token of the sequence has position lens[0].
+ * With k = v = NULL the entries are filled on the device instead, element x
+ * of the pool getting (fmix32(x) mod 256 - 128) / 64 (fmix32 = the 32-bit
+ * MurmurHash3 finaliser): for long caches whose values do not matter, such
+ * as throughput runs.
  * Errors: INVALID_ARG, DUPLICATE_SEQ, CAPACITY, SEQ_TOO_LONG, OUT_OF_PAGES,
  * CUDA, NO_DEVICE. */
 int tlf_load_cache(tlf_ctx* ctx, uint64_t seq_id, const int32_t* lens, const int32_t* positions,

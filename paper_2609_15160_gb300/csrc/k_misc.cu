@@ -224,6 +224,49 @@ __global__ void k_scatter_cache(ModelDims md, int slot, int r, int n, const T* _
   if (threadIdx.x == 0) pos_table[(size_t)page * ps + off] = positions[e];
 }
 
+// K/V of entries e < n of loop r filled with a counter-based pattern: value =
+// (h(x) mod 256 - 128) / 64 for x the element's index in the pool, with h the
+// 32-bit integer finaliser of MurmurHash3 (multiples of 1/64 in [-2, 2),
+// exact in bf16). Used to restore long caches whose values do not matter.
+__device__ __forceinline__ uint32_t fmix32(uint32_t h) {
+  h ^= h >> 16;
+  h *= 0x85ebca6bu;
+  h ^= h >> 13;
+  h *= 0xc2b2ae35u;
+  h ^= h >> 16;
+  return h;
+}
+
+template <typename T>
+__global__ void k_fill_cache(ModelDims md, int slot, int r, int n, const int* __restrict__ positions,
+                             const int* __restrict__ page_table, T* pool, int* pos_table) {
+  const int e = blockIdx.x;
+  if (e >= n) return;
+  const int ps = md.page_size, hd = md.hd;
+  const int page = page_table[((size_t)slot * md.M + r) * md.max_pages + e / ps];
+  if (page < 0 || page >= md.n_pages) return;
+  const int off = e % ps;
+  T* pg = pool + (size_t)page * md.page_elems;
+  const int per = md.J * md.Hkv * hd;
+  for (int t = threadIdx.x; t < 2 * per; t += blockDim.x) {
+    const int kv = t / per, rem = t % per;
+    const int jj = rem / (md.Hkv * hd), rem2 = rem % (md.Hkv * hd), h = rem2 / hd, i = rem2 % hd;
+    const size_t idx = ((size_t)(jj * 2 + kv) * md.Hkv + h) * ps * hd + (size_t)off * hd + i;
+    const uint32_t x = fmix32((uint32_t)((size_t)page * md.page_elems + idx));
+    pg[idx] = from_f32<T>((float)((int)(x & 255u) - 128) / 64.f);
+  }
+  if (threadIdx.x == 0) pos_table[(size_t)page * ps + off] = positions[e];
+}
+
+void launch_fill_cache(const ModelDims& md, int slot, int r, int n, const int* positions, const int* page_table,
+                       void* pool, int* pos_table, cudaStream_t st) {
+  if (n <= 0) return;
+  if (md.dtype == 1)
+    k_fill_cache<bf16><<<n, 256, 0, st>>>(md, slot, r, n, positions, page_table, (bf16*)pool, pos_table);
+  else
+    k_fill_cache<float><<<n, 256, 0, st>>>(md, slot, r, n, positions, page_table, (float*)pool, pos_table);
+}
+
 void launch_scatter_cache(const ModelDims& md, int slot, int r, int n, const void* k, const void* v,
                           const int* positions, const int* page_table, void* pool, int* pos_table, cudaStream_t st) {
   if (n <= 0) return;

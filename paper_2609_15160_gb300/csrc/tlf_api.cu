@@ -945,7 +945,8 @@ extern "C" int tlf_prefill(tlf_ctx* ctx, int32_t n_seqs, const uint64_t* seq_ids
 extern "C" int tlf_load_cache(tlf_ctx* ctx, uint64_t seq_id, const int32_t* lens, const int32_t* positions,
                               const void* k, const void* v) {
   if (!ctx) return TLF_ERR_INVALID_ARG;
-  if (!lens || !positions || !k || !v) return fail(ctx, TLF_ERR_INVALID_ARG, "NULL argument");
+  if (!lens || !positions || (!k) != (!v)) return fail(ctx, TLF_ERR_INVALID_ARG, "NULL argument");
+  const bool fill = (k == nullptr);  // entries filled on the device with a counter-based pattern
   const int M = ctx->md.M, ps = ctx->md.page_size;
   if (ctx->seq_slot.count(seq_id)) return fail(ctx, TLF_ERR_DUPLICATE_SEQ, "sequence %llu is live", (unsigned long long)seq_id);
   if (ctx->free_slots.empty()) return fail(ctx, TLF_ERR_CAPACITY, "no free sequence slot");
@@ -996,18 +997,28 @@ extern "C" int tlf_load_cache(tlf_ctx* ctx, uint64_t seq_id, const int32_t* lens
   void *dk = nullptr, *dv = nullptr;
   int* dp = nullptr;
   if (e == cudaSuccess && lens[0] > 0) {
-    e = cudaMalloc(&dk, (size_t)lens[0] * per * ctx->eb);
-    if (e == cudaSuccess) e = cudaMalloc(&dv, (size_t)lens[0] * per * ctx->eb);
+    if (!fill) {
+      e = cudaMalloc(&dk, (size_t)lens[0] * per * ctx->eb);
+      if (e == cudaSuccess) e = cudaMalloc(&dv, (size_t)lens[0] * per * ctx->eb);
+    }
     if (e == cudaSuccess) e = cudaMalloc(&dp, (size_t)lens[0] * 4);
   }
   for (int r = 0; r < M && e == cudaSuccess; ++r) {
     if (lens[r] == 0) continue;
-    e = cudaMemcpy(dk, (const uint8_t*)k + offs[r] * per * ctx->eb, (size_t)lens[r] * per * ctx->eb, cudaMemcpyHostToDevice);
-    if (e == cudaSuccess)
-      e = cudaMemcpy(dv, (const uint8_t*)v + offs[r] * per * ctx->eb, (size_t)lens[r] * per * ctx->eb, cudaMemcpyHostToDevice);
+    if (!fill) {
+      e = cudaMemcpy(dk, (const uint8_t*)k + offs[r] * per * ctx->eb, (size_t)lens[r] * per * ctx->eb,
+                     cudaMemcpyHostToDevice);
+      if (e == cudaSuccess)
+        e = cudaMemcpy(dv, (const uint8_t*)v + offs[r] * per * ctx->eb, (size_t)lens[r] * per * ctx->eb,
+                       cudaMemcpyHostToDevice);
+    }
     if (e == cudaSuccess) e = cudaMemcpy(dp, positions + offs[r], (size_t)lens[r] * 4, cudaMemcpyHostToDevice);
     if (e == cudaSuccess) {
-      launch_scatter_cache(ctx->md, slot, r, lens[r], dk, dv, dp, ctx->d_page_table, ctx->d_pool, ctx->d_pos_table, 0);
+      if (fill)
+        launch_fill_cache(ctx->md, slot, r, lens[r], dp, ctx->d_page_table, ctx->d_pool, ctx->d_pos_table, 0);
+      else
+        launch_scatter_cache(ctx->md, slot, r, lens[r], dk, dv, dp, ctx->d_page_table, ctx->d_pool,
+                             ctx->d_pos_table, 0);
       e = cudaDeviceSynchronize();
     }
   }

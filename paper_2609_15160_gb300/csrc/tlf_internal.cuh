@@ -387,6 +387,8 @@ void launch_final(const ModelDims& md, const StepDev& s, int B, const float* gai
 void launch_scatter_cache(const ModelDims& md, int slot, int r, int n, const void* k, const void* v,
                           const int* positions, const int* page_table, void* pool, int* pos_table,
                           cudaStream_t st);
+void launch_fill_cache(const ModelDims& md, int slot, int r, int n, const int* positions, const int* page_table,
+                       void* pool, int* pos_table, cudaStream_t st);
 
 // Kernel-level attention operation (tlf_attn_decode): scratch layout and launch.
 struct AttnOpLayout {

@@ -281,6 +281,15 @@ def make_cache_snapshot(m: ModelConfig, length: int, seed: int,
     return {"depths": np.asarray(depths, dtype=np.int32), "positions": pos, "k": ks, "v": vs}
 
 
+def make_cache_positions(m: ModelConfig, length: int, seed: int,
+                         depths: Optional[np.ndarray] = None) -> dict:
+    """Only the positions of a cache snapshot (values to be filled on the device)."""
+    if depths is None:
+        depths = sample_depths(m.depth_probs, m.max_loops, length, seed)
+    return {"depths": np.asarray(depths, dtype=np.int32),
+            "positions": [np.nonzero(depths >= r)[0].astype(np.int32) for r in range(1, m.max_loops + 1)]}
+
+
 def make_attn_problem(n: int, lens, hq: int, hkv: int, hd: int, n_layers: int = 2, layer: int = 1,
                       dtype: str = "bf16", seed: int = 0, spare_pages: int = 3, page_size: int = 64) -> dict:
     """Inputs of the kernel-level attention operation on paged caches.

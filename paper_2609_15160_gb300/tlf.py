@@ -204,9 +204,12 @@ def tlf_release(ctx, seq_id: int):
     _check(load_library().tlf_release(ctx, C.c_uint64(seq_id)), ctx)
 
 
-def tlf_load_cache(ctx, seq_id: int, lens: np.ndarray, positions: np.ndarray, k: np.ndarray, v: np.ndarray):
+def tlf_load_cache(ctx, seq_id: int, lens: np.ndarray, positions: np.ndarray, k: Optional[np.ndarray],
+                   v: Optional[np.ndarray]):
+    """k = v = None: entries are filled on the device (see include/tlf.h)."""
     _check(load_library().tlf_load_cache(ctx, C.c_uint64(seq_id), _ptr(lens, C.c_int32), _ptr(positions, C.c_int32),
-                                         k.ctypes.data, v.ctypes.data), ctx)
+                                         None if k is None else k.ctypes.data,
+                                         None if v is None else v.ctypes.data), ctx)
 
 
 def attn_args(n, n_heads, n_kv_heads, head_dim, n_layers, layer, dtype, max_pages, n_pages, q, pool, page_table,
@@ -299,9 +302,13 @@ class Context:
         tlf_release(self.handle, seq_id)
 
     def load_cache(self, seq_id: int, snapshot: dict):
-        """snapshot: synth.make_cache_snapshot output (values exact in the model dtype)."""
+        """snapshot: synth.make_cache_snapshot output (values exact in the model dtype); without
+        "k"/"v" entries (synth.make_cache_positions) the values are filled on the device."""
         lens = np.array([len(p) for p in snapshot["positions"]], dtype=np.int32)
         pos = np.ascontiguousarray(np.concatenate(snapshot["positions"]).astype(np.int32))
+        if "k" not in snapshot:
+            tlf_load_cache(self.handle, seq_id, lens, pos, None, None)
+            return
         k = np.concatenate(snapshot["k"]).astype(np.float32)
         v = np.concatenate(snapshot["v"]).astype(np.float32)
         tlf_load_cache(self.handle, seq_id, lens, pos, _matrix(k, self.model.dtype), _matrix(v, self.model.dtype))

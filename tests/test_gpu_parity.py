@@ -274,6 +274,24 @@ def test_profile_counters(tlf):
         assert abs(by - want) < 1e-6 * want
 
 
+def test_device_filled_restore(tlf):
+    """tlf_load_cache without values: lengths and positions as given, values on the 1/64 grid in [-2, 2)."""
+    m = _small()
+    w = synth.make_weights(m)
+    snap = synth.make_cache_positions(m, 300, seed=5)
+    with tlf.Context(m, w, max_seqs=1, max_batch=1, max_seq_len=400) as ctx:
+        ctx.load_cache(9, snap)
+        for r in range(1, m.max_loops + 1):
+            assert ctx.cache_len(9, r) == len(snap["positions"][r - 1])
+            p, k, v = ctx.read_cache(9, r, m.n_layers - 1)
+            np.testing.assert_array_equal(p, snap["positions"][r - 1])
+            for a in (k, v):
+                if a.size:
+                    assert np.all(a * 64 == np.round(a * 64)) and a.min() >= -2 and a.max() < 2 and a.std() > 0.5
+        lg, loops, _ = ctx.decode_step([9], [3])
+        assert np.all(np.isfinite(lg))
+
+
 def test_decode_step_is_deterministic(tlf):
     """Two contexts fed the same inputs produce bitwise identical logits and caches.
 
