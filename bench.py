@@ -7,8 +7,9 @@ compaction, every loop's shared block on its active tokens, recursion-wise
 attention, LM head). Default workload: the long-context GQA model (d 2048,
 16 q / 8 kv heads x 128, 2 layers, ffn 5504, M = 6) with batch 16 at 32768
 tokens of context, the configuration the attention bandwidth target is set on.
-Sequences start from restored synthetic cache snapshots whose per-loop lengths
-follow the model's depth distribution (prefill is not part of the step).
+The sequences' caches are built by prefilling the seeded prompts through the
+library before timing (prefill is not part of the step; its time is reported);
+--prefill snapshot restores synthetic caches instead.
 
 Prints one JSON line. ``value`` is decode tokens/s over all ranks, timed with
 CUDA events on the launching stream with logits left on the device; ``e2e``
@@ -174,7 +175,7 @@ def setup_workload(T, wl, rank: int, gemm_impl="auto", prefill="auto", extra_tok
     prompts = synth.make_prompts(wl)
     lengths = [len(p) for p in prompts]
     steps_cap = max(wl.decode_steps, extra_tokens) + 64
-    use_snapshot = prefill == "snapshot" or (prefill == "auto" and max(lengths) > 4096)
+    use_snapshot = prefill == "snapshot"  # default: real (batched) prefill through the library
     ids = [rank * 100000 + b for b in range(B)]
     if use_snapshot:
         # uniform lengths: two distinct host snapshots (values uploaded); ragged lengths: one
@@ -201,7 +202,10 @@ def setup_workload(T, wl, rank: int, gemm_impl="auto", prefill="auto", extra_tok
             ctx.load_cache(ids[b], snaps[b])
     else:
         forced = None if wl.forced_loops is None else [np.full(len(p), wl.forced_loops, np.int32) for p in prompts]
+        t_pf = time.time()
         ctx.prefill(ids, prompts, forced=forced, logits=False)
+        ctx.prefill_seconds = time.time() - t_pf
+        ctx.prefill_tokens = sum(len(p) for p in prompts)
     if snaps is None:
         how = "prefill through the library"
     elif "k" in snaps[0]:
@@ -333,6 +337,9 @@ def run_ours(args):
             "gpu_launches": int(launches),
             "kernel_ms_per_step_profiled": {k: round(v, 4) for k, v in breakdown.items()},
             "setup_s": setup_s,
+            "prefill": ({"tokens": ctx.prefill_tokens, "seconds": ctx.prefill_seconds,
+                         "tokens_per_s": ctx.prefill_tokens / ctx.prefill_seconds}
+                        if hasattr(ctx, "prefill_seconds") else None),
         }
         if clk:
             line["clocks"] = clk
@@ -397,9 +404,61 @@ def run_attn_op(args):
                                    "algorithmic_bytes_per_call": kv_bytes + io_bytes}}))
 
 
+def run_ttft(args):
+    """Time to first token: one prompt of each length through tlf_prefill (logits of its last token).
+
+    The paper reports TTFT for prompts of 128, 512, 1024 and 2048 tokens (Fig. 4d); the prompts here are
+    seeded uniform random ids on the chosen workload's model. Also reports the prefill throughput of the
+    workload's whole batch of prompts (--full).
+    """
+    import torch
+
+    from paper_2609_15160_gb300 import tlf as T
+
+    T.load_library()
+    wl = synth.get_config(args.config)
+    m = wl.model
+    w = synth.make_weights(m)
+    lengths = [int(x) for x in args.ttft_lengths.split(",")]
+    B = wl.batch
+    full_prompts = synth.make_prompts(wl) if args.full else []
+    max_len = max(lengths + [len(p) for p in full_prompts])
+    n_pages = max(len(full_prompts), 1) * m.max_loops * ((max_len + 63) // 64 + 2) + 64
+    ctx = T.Context(m, w, max_seqs=max(B, 2), max_batch=min(B, 256), max_seq_len=max_len + 8,
+                    kv_pool_pages=n_pages)
+    rng = np.random.default_rng(4)
+    out = []
+    for L in lengths:
+        prompt = rng.integers(0, m.vocab, size=L).astype(np.int32)
+        times = []
+        for it in range(args.warmup + args.steps):
+            torch.cuda.synchronize()
+            t0 = time.perf_counter()
+            ctx.prefill([7], [prompt])
+            times.append(time.perf_counter() - t0)
+            ctx.release(7)
+        ms = 1e3 * float(np.median(times[args.warmup:]))
+        out.append({"prompt_len": L, "ttft_ms": ms})
+    line = {"metric": "ttft_ms", "unit": "ms", "higher_is_better": False, "config": {"workload": DESCR[args.config],
+            "model": args.config, "dtype": m.dtype, "data": "synthetic uniform random prompts"}, "ttft": out}
+    if args.full:
+        torch.cuda.synchronize()
+        t0 = time.perf_counter()
+        ctx.prefill(list(range(100, 100 + B)), full_prompts, logits=False)
+        torch.cuda.synchronize()
+        sec = time.perf_counter() - t0
+        ntok = sum(len(p) for p in full_prompts)
+        line["full_prefill"] = {"sequences": B, "tokens": ntok, "seconds": sec, "tokens_per_s": ntok / sec}
+    print(json.dumps(line))
+    ctx.close()
+
+
 def main():
     ap = argparse.ArgumentParser()
-    ap.add_argument("--op", default=None, choices=["attn"], help="time one kernel-level operation alone")
+    ap.add_argument("--op", default=None, choices=["attn", "ttft"],
+                    help="time one operation alone: the attention kernels, or prefill (time to first token)")
+    ap.add_argument("--ttft-lengths", default="128,512,1024,2048")
+    ap.add_argument("--full", action="store_true", help="--op ttft: also prefill the workload's whole batch")
     ap.add_argument("--batch", type=int, default=16)
     ap.add_argument("--context", type=int, default=32768)
     ap.add_argument("--hq", type=int, default=16, help="--op attn: query heads")
@@ -419,6 +478,8 @@ def main():
         args.warmup = 3
     if args.op == "attn":
         run_attn_op(args)
+    elif args.op == "ttft":
+        run_ttft(args)
     elif args.impl == "reference":
         run_reference(args)
     else:

@@ -93,7 +93,7 @@ typedef struct tlf_config {
   int32_t page_size;    /* tokens per KV page, multiple of 16 (64 is a good default) */
   int32_t gemm_impl;    /* tlf_gemm_impl */
   int32_t host_only;    /* 1: allocate nothing on a GPU; only validation and bookkeeping run */
-  int32_t reserved0;
+  int32_t prefill_chunk;/* prompt tokens per batched-prefill chunk (bf16 models); 0 = 8192 */
   int64_t kv_pool_pages;/* pages in the KV pool; 0 = max_seqs * max_loops * ceil(max_seq_len / page_size) */
 } tlf_config;
 

@@ -72,7 +72,7 @@ __device__ __forceinline__ void cluster_sum4(const uint32_t* pb, int S, int f, i
 }
 
 template <int NT>
-__device__ void cluster_epilogue(const GemmArgs& a, float* red, int* colinfo, int m0, int n) {
+__device__ void cluster_epilogue(const GemmArgs& a, float* red, int* colinfo, int m0, int n, int tok0) {
   const int S = a.splits;
   const int rank = (int)cluster_ctarank();
   const int per = (n + S - 1) / S;
@@ -92,7 +92,7 @@ __device__ void cluster_epilogue(const GemmArgs& a, float* red, int* colinfo, in
 #pragma unroll
         for (int q = 0; q < 4; ++q)
           if (c + q < c1) {
-            const int row = a.idx ? a.idx[c + q] : c + q;
+            const int row = a.idx ? a.idx[tok0 + c + q] : tok0 + c + q;
             atomicAdd(a.resid + (size_t)row * a.ldr + col, sm[q]);  // the only writer of this element
           }
       }
@@ -108,7 +108,7 @@ __device__ void cluster_epilogue(const GemmArgs& a, float* red, int* colinfo, in
 #pragma unroll
         for (int q = 0; q < 4; ++q)
           if (c + q < c1)
-            reinterpret_cast<bf16*>(a.U)[(size_t)(c + q) * a.md.ff + gf] =
+            reinterpret_cast<bf16*>(a.U)[(size_t)(tok0 + c + q) * a.md.ff + gf] =
                 __float2bfloat16_rn(g[q] / (1.f + expf(-g[q])) * u[q]);
       }
     return;
@@ -121,19 +121,26 @@ __device__ void cluster_epilogue(const GemmArgs& a, float* red, int* colinfo, in
   int* ci_page = colinfo + NT;
   int* ci_off = colinfo + 2 * NT;
   for (int t = tid; t < c1 - c0; t += blockDim.x) {
-    const int c = c0 + t;
-    const int b = s.idx[a.r * md.max_batch + c];
-    const int slot = s.slots[b];
-    const int L = s.len[slot * md.M + a.r];
+    const int row = tok0 + c0 + t;
+    int slot, L, pos;
+    if (a.row_cslot) {  // prefill: per-row sequence slot, cache slot and position from the plan
+      slot = a.row_slot[row];
+      L = a.row_cslot[row];
+      pos = a.row_pos[row];
+    } else {            // decode: the token appends at the end of its loop-r cache
+      slot = s.slots[s.idx[a.r * md.max_batch + row]];
+      L = s.len[slot * md.M + a.r];
+      pos = s.len[slot * md.M];  // every token runs loop 1: its length is the token count
+    }
     int page = s.page_table[((size_t)slot * md.M + a.r) * md.max_pages + L / ps];
     if (page < 0 || page >= md.n_pages) {
       atomicOr(s.err, DEVERR_INDEX);
       page = -1;
     }
-    ci_pos[t] = s.len[slot * md.M];  // every token runs loop 1: its length is the token count
+    ci_pos[t] = pos;
     ci_page[t] = page;
     ci_off[t] = L % ps;
-    if (a.j == 0 && page >= 0) s.pos_table[(size_t)page * ps + L % ps] = ci_pos[t];
+    if (a.j == 0 && page >= 0) s.pos_table[(size_t)page * ps + L % ps] = pos;
   }
   __syncthreads();
   const int gfeat = m0 + tid;
@@ -160,7 +167,7 @@ __device__ void cluster_epilogue(const GemmArgs& a, float* red, int* colinfo, in
         sincosf((float)ang, &sn, &cs);
         const float r0 = x0[q] * cs - x1[q] * sn, r1 = x0[q] * sn + x1[q] * cs;
         if (is_q) {
-          float* qo = a.Q + ((size_t)cc * md.Hq + h) * hd;
+          float* qo = a.Q + ((size_t)(tok0 + cc) * md.Hq + h) * hd;
           qo[i] = r0;
           qo[i + half] = r1;
         } else if (ci_page[cc - c0] >= 0) {
@@ -207,12 +214,14 @@ __global__ void __launch_bounds__(128) k_gemm_tc(const __grid_constant__ CUtenso
   // The token count comes from the plan kernel, which completed before this
   // grid was launched (every kernel triggers its successor only after its own
   // wait), so it is read before pdl_wait(), bypassing L1.
-  const int n = a.n_dev ? __ldcg(a.n_dev) : a.n_host;
-  if (n <= 0) {
+  const int n_all = a.n_dev ? __ldcg(a.n_dev) : a.n_host;
+  const int tok0 = blockIdx.z * NT;  // token tile of this CTA (prefill has many)
+  if (n_all <= tok0) {
     pdl_wait();
     pdl_trigger();
     return;
   }
+  const int n = min(NT, n_all - tok0);      // token columns of this tile
   const int ncols = ((n + 15) / 16) * 16;  // MMA N: multiple of 16, <= NT
   const int m0 = blockIdx.x * TC_BM;
   const int split = blockIdx.y;
@@ -254,7 +263,7 @@ __global__ void __launch_bounds__(128) k_gemm_tc(const __grid_constant__ CUtenso
     }
     pdl_wait();
     pdl_trigger();
-    for (int i = 0; i < pre; ++i) tma_load_2d(smem_u32(sB + i * B_BYTES), &mapX, (kb0 + i) * TC_BK, 0, full(i));
+    for (int i = 0; i < pre; ++i) tma_load_2d(smem_u32(sB + i * B_BYTES), &mapX, (kb0 + i) * TC_BK, tok0, full(i));
     for (int i = pre; i < nk; ++i) {
       const int st = i % TC_STAGES;
       const uint32_t ph = (uint32_t)(i / TC_STAGES) & 1u;
@@ -262,7 +271,7 @@ __global__ void __launch_bounds__(128) k_gemm_tc(const __grid_constant__ CUtenso
       mbar_arrive_expect_tx(full(st), A_BYTES + B_BYTES);
       const int kx = (kb0 + i) * TC_BK;
       tma_load_2d(smem_u32(sA + st * A_BYTES), &mapW, kx, m0, full(st));
-      tma_load_2d(smem_u32(sB + st * B_BYTES), &mapX, kx, 0, full(st));
+      tma_load_2d(smem_u32(sB + st * B_BYTES), &mapX, kx, tok0, full(st));
     }
   } else {
     pdl_wait();
@@ -316,7 +325,7 @@ __global__ void __launch_bounds__(128) k_gemm_tc(const __grid_constant__ CUtenso
     __syncthreads();
     if (warp == 0) tmem_dealloc(tmem, TMEM_COLS);
     cluster_sync_all();  // every partner's tile is staged
-    cluster_epilogue<NT>(a, red, colinfo, m0, n);
+    cluster_epilogue<NT>(a, red, colinfo, m0, n, tok0);
     __syncwarp();
     cluster_sync_all();  // partners have finished reading this CTA's tile
     return;
@@ -334,7 +343,7 @@ __global__ void __launch_bounds__(128) k_gemm_tc(const __grid_constant__ CUtenso
       if (col < a.N) {
 #pragma unroll
         for (int i = 0; i < 16; ++i)
-          if (c0 + i < n && (nk > 0 || a.epi == EPI_PARTIAL)) gemm_write(a, split, c0 + i, col, v[i]);
+          if (c0 + i < n && (nk > 0 || a.epi == EPI_PARTIAL)) gemm_write(a, split, tok0 + c0 + i, col, v[i]);
       }
     }
   }
@@ -353,7 +362,7 @@ static void launch_tc_nt(const CUtensorMap* mapW, const CUtensorMap* mapX, const
     cudaFuncSetAttribute(k_gemm_tc<NT>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
     attr_set = true;
   }
-  dim3 grid((a.N + TC_BM - 1) / TC_BM, a.splits);
+  dim3 grid((a.N + TC_BM - 1) / TC_BM, a.splits, a.tok_tiles > 0 ? a.tok_tiles : 1);
   if (a.epi < EPI_CL_RESID) {
     launch_k(k_gemm_tc<NT>, grid, 128, smem, st, *mapW, *mapX, a);
     return;

@@ -107,6 +107,25 @@ struct tlf_ctx {
   uint32_t* h_err = nullptr;
   int s_qkv = 1, s_o = 1, s_gu = 1, s_d = 1, split_cap = 8;
 
+  // batched prefill (bf16 models): chunk workspaces, allocated on first use
+  int pf_C = 0, pf_Smax = 0;
+  size_t pf_in_ints = 0;
+  int* d_pf_in = nullptr;
+  int* h_pf_in = nullptr;
+  int* d_pf_m = nullptr;
+  float* d_pf_margin = nullptr;
+  float* d_pf_H = nullptr;
+  void* d_pf_X = nullptr;
+  float* d_pf_Q = nullptr;
+  void* d_pf_O = nullptr;
+  void* d_pf_U = nullptr;
+  CUtensorMap pf_map_X, pf_map_O, pf_map_U;
+  int *d_pf_idx = nullptr, *d_pf_n = nullptr, *d_pf_row_slot = nullptr, *d_pf_row_cslot = nullptr,
+      *d_pf_row_pos = nullptr, *d_pf_first = nullptr, *d_pf_cnt = nullptr, *d_pf_s0 = nullptr,
+      *d_pf_tile_base = nullptr;
+  int* h_pf_m = nullptr;
+  float pf_last_ms = 0.f;
+
   // profiling
   bool profiling = false;
   float last_attn_ms = 0.f;
@@ -199,6 +218,8 @@ extern "C" int tlf_validate_config(const tlf_config* c, char* msg, size_t msg_le
   if (c->page_size != 64) return bad("page_size must be 64");
   if (c->gemm_impl != TLF_GEMM_AUTO && c->gemm_impl != TLF_GEMM_SIMT) return bad("unknown gemm_impl");
   if (c->kv_pool_pages < 0) return bad("kv_pool_pages must be >= 0");
+  if (c->prefill_chunk < 0 || (c->prefill_chunk > 0 && c->prefill_chunk < 64))
+    return bad("prefill_chunk must be 0 (default) or >= 64");
   if (msg && msg_len) snprintf(msg, msg_len, "ok");
   return TLF_OK;
 }
@@ -483,6 +504,11 @@ extern "C" void tlf_destroy(tlf_ctx* ctx) {
     if (ctx->h_err) cudaFreeHost(ctx->h_err);
     for (auto e : ctx->events) if (e) cudaEventDestroy(e);
     for (auto& g : ctx->graphs) cudaGraphExecDestroy(g.exec);
+    f(ctx->d_pf_in); f(ctx->d_pf_m); f(ctx->d_pf_margin); f(ctx->d_pf_H); f(ctx->d_pf_X); f(ctx->d_pf_Q);
+    f(ctx->d_pf_O); f(ctx->d_pf_U); f(ctx->d_pf_idx); f(ctx->d_pf_n); f(ctx->d_pf_row_slot); f(ctx->d_pf_row_cslot);
+    f(ctx->d_pf_row_pos); f(ctx->d_pf_first); f(ctx->d_pf_cnt); f(ctx->d_pf_s0); f(ctx->d_pf_tile_base);
+    if (ctx->h_pf_in) cudaFreeHost(ctx->h_pf_in);
+    if (ctx->h_pf_m) cudaFreeHost(ctx->h_pf_m);
     if (ctx->cap_stream) cudaStreamDestroy(ctx->cap_stream);
   }
   delete ctx;
@@ -867,6 +893,270 @@ extern "C" int tlf_decode_step(tlf_ctx* ctx, int32_t batch, const uint64_t* seq_
   return TLF_OK;
 }
 
+// ----------------------------------------------------------------------------
+// batched prefill (tensor-core models)
+// ----------------------------------------------------------------------------
+static int ensure_prefill_buffers(tlf_ctx* ctx) {
+  if (ctx->pf_C) return TLF_OK;
+  const ModelDims& md = ctx->md;
+  int C = ctx->cfg.prefill_chunk > 0 ? ctx->cfg.prefill_chunk : 8192;
+  C = (C + 255) / 256 * 256;
+  const int Smax = std::min(1024, std::min(C, ctx->cfg.max_seqs));
+  const int M = md.M, d = md.d;
+  const size_t max_upd = (size_t)M * (C / 64 + 2 * (size_t)Smax);
+  ctx->pf_in_ints = 1 + 4 * (size_t)C + 2 * (size_t)Smax + 2 * max_upd;
+  int rc;
+  if ((rc = dev_alloc(ctx, &ctx->d_pf_in, ctx->pf_in_ints * 4, "prefill inputs"))) return rc;
+  CK(ctx, cudaMallocHost((void**)&ctx->h_pf_in, ctx->pf_in_ints * 4));
+  CK(ctx, cudaMallocHost((void**)&ctx->h_pf_m, (size_t)C * 4));
+  if ((rc = dev_alloc(ctx, &ctx->d_pf_m, (size_t)C * 4, "prefill m"))) return rc;
+  if ((rc = dev_alloc(ctx, &ctx->d_pf_margin, (size_t)C * 4, "prefill margin"))) return rc;
+  if ((rc = dev_alloc(ctx, &ctx->d_pf_H, (size_t)C * d * 4, "prefill H"))) return rc;
+  if ((rc = dev_alloc(ctx, &ctx->d_pf_X, (size_t)C * d * 2, "prefill X"))) return rc;
+  if ((rc = dev_alloc(ctx, &ctx->d_pf_Q, (size_t)C * md.q_dim * 4, "prefill Q"))) return rc;
+  if ((rc = dev_alloc(ctx, &ctx->d_pf_O, (size_t)C * md.q_dim * 2, "prefill O"))) return rc;
+  if ((rc = dev_alloc(ctx, &ctx->d_pf_U, (size_t)C * md.ff * 2, "prefill U"))) return rc;
+  if ((rc = dev_alloc(ctx, &ctx->d_pf_idx, (size_t)M * C * 4, "prefill idx"))) return rc;
+  if ((rc = dev_alloc(ctx, &ctx->d_pf_row_slot, (size_t)M * C * 4, "prefill rows"))) return rc;
+  if ((rc = dev_alloc(ctx, &ctx->d_pf_row_cslot, (size_t)M * C * 4, "prefill rows"))) return rc;
+  if ((rc = dev_alloc(ctx, &ctx->d_pf_row_pos, (size_t)M * C * 4, "prefill rows"))) return rc;
+  if ((rc = dev_alloc(ctx, &ctx->d_pf_n, (size_t)M * 4, "prefill n"))) return rc;
+  if ((rc = dev_alloc(ctx, &ctx->d_pf_first, (size_t)M * Smax * 4, "prefill seqs"))) return rc;
+  if ((rc = dev_alloc(ctx, &ctx->d_pf_cnt, (size_t)M * Smax * 4, "prefill seqs"))) return rc;
+  if ((rc = dev_alloc(ctx, &ctx->d_pf_s0, (size_t)M * Smax * 4, "prefill seqs"))) return rc;
+  if ((rc = dev_alloc(ctx, &ctx->d_pf_tile_base, (size_t)M * (Smax + 1) * 4, "prefill tiles"))) return rc;
+  CK(ctx, cudaMemset(ctx->d_pf_X, 0, (size_t)C * d * 2));
+  CK(ctx, cudaMemset(ctx->d_pf_O, 0, (size_t)C * md.q_dim * 2));
+  CK(ctx, cudaMemset(ctx->d_pf_U, 0, (size_t)C * md.ff * 2));
+  if (!make_map(&ctx->pf_map_X, ctx->d_pf_X, C, d, d, 256) ||
+      !make_map(&ctx->pf_map_O, ctx->d_pf_O, C, md.q_dim, md.q_dim, 256) ||
+      !make_map(&ctx->pf_map_U, ctx->d_pf_U, C, md.ff, md.ff, 256))
+    return fail(ctx, TLF_ERR_CUDA, "cuTensorMapEncodeTiled failed for a prefill buffer");
+  ctx->pf_C = C;
+  ctx->pf_Smax = Smax;
+  return TLF_OK;
+}
+
+static void gemm_pf(tlf_ctx* ctx, const DeviceMat& W, const CUtensorMap* xmap, GemmArgs a, cudaStream_t st) {
+  a.N = W.N;
+  a.K = W.K;
+  a.err = ctx->d_err;
+  a.splits = 1;
+  a.max_rows = ctx->pf_C;
+  a.tok_tiles = ctx->pf_C / 256;
+  launch_gemm_tc(&W.map, xmap, 256, a, st);
+}
+
+// Prompts of the (already created) sequences slot_of[0..n), chunk by chunk: every chunk is routed,
+// runs all loops on its gathered tokens (Eq. 6-7) with causal attention over each sequence's
+// loop caches (Eq. 10), and appends its k, v at the following cache slots (Eq. 11, App. B).
+static int prefill_batched(tlf_ctx* ctx, int n_seqs, const int* slot_of, const int32_t* offsets,
+                           const int32_t* tokens, const int32_t* forced, float* last_logits, bool logits_dev,
+                           int32_t* loops, cudaStream_t st) {
+  int rc = ensure_prefill_buffers(ctx);
+  if (rc) return rc;
+  const ModelDims& md = ctx->md;
+  const int M = md.M, J = md.J, C = ctx->pf_C, Smax = ctx->pf_Smax, ps = md.page_size, maxB = md.max_batch;
+  struct Seg {
+    int s, start, count;
+  };
+  int s_next = 0, pos_next = 0;
+  while (s_next < n_seqs) {
+    std::vector<Seg> segs;
+    int T = 0;
+    while (s_next < n_seqs && T < C && (int)segs.size() < Smax) {
+      const int len = offsets[s_next + 1] - offsets[s_next];
+      const int take = std::min(len - pos_next, C - T);
+      segs.push_back({s_next, pos_next, take});
+      T += take;
+      pos_next += take;
+      if (pos_next == len) {
+        ++s_next;
+        pos_next = 0;
+      }
+    }
+    const int S = (int)segs.size();
+    // pages: worst case (every chunk token runs every loop); trimmed once the loop counts are known
+    size_t need = 0;
+    for (const Seg& g : segs)
+      for (int r = 0; r < M; ++r) {
+        const int L = ctx->h_len[(size_t)slot_of[g.s] * M + r];
+        for (int p = L / ps; p <= (L + g.count - 1) / ps; ++p)
+          if (pt_at(ctx, slot_of[g.s], r, p) < 0) ++need;
+      }
+    if (need > ctx->free_pages.size())
+      return fail(ctx, TLF_ERR_OUT_OF_PAGES, "prefill chunk needs %zu KV pages, %zu free", need,
+                  ctx->free_pages.size());
+    int* h = ctx->h_pf_in;
+    int* h_upd = h + 1 + 4 * C + 2 * Smax;
+    int nu = 0;
+    for (const Seg& g : segs)
+      for (int r = 0; r < M; ++r) {
+        const int slot = slot_of[g.s];
+        const int L = ctx->h_len[(size_t)slot * M + r];
+        for (int p = L / ps; p <= (L + g.count - 1) / ps; ++p) {
+          int& e = pt_at(ctx, slot, r, p);
+          if (e < 0) {
+            e = ctx->free_pages.back();
+            ctx->free_pages.pop_back();
+            h_upd[2 * nu] = (int)(((size_t)slot * M + r) * md.max_pages + p);
+            h_upd[2 * nu + 1] = e;
+            ++nu;
+          }
+        }
+      }
+    h[0] = nu;
+    std::vector<int> ending;  // prompts whose last token is in this chunk
+    int nend = 0;
+    for (int si = 0, t = 0; si < S; ++si) {
+      const Seg& g = segs[si];
+      for (int i = 0; i < g.count; ++i, ++t) {
+        const int gi = offsets[g.s] + g.start + i;
+        h[1 + t] = tokens[gi];
+        h[1 + C + t] = forced ? forced[gi] : -1;
+        h[1 + 2 * C + t] = si;
+        h[1 + 3 * C + t] = g.start + i;
+      }
+      h[1 + 4 * C + si] = slot_of[g.s];
+      if (g.start + g.count == offsets[g.s + 1] - offsets[g.s]) {
+        h[1 + 4 * C + Smax + nend++] = t - 1;
+        ending.push_back(g.s);
+      }
+    }
+    CK(ctx, cudaMemcpyAsync(ctx->d_pf_in, h, (size_t)(1 + 4 * C + 2 * Smax + 2 * nu) * 4, cudaMemcpyHostToDevice, st));
+
+    StepDev sr{};
+    sr.tokens = ctx->d_pf_in + 1;
+    sr.forced = ctx->d_pf_in + 1 + C;
+    sr.m = ctx->d_pf_m;
+    sr.margin = ctx->d_pf_margin;
+    sr.H = ctx->d_pf_H;
+    sr.page_table = ctx->d_page_table;
+    sr.err = ctx->d_err;
+    launch_router(md, sr, T, ctx->d_emb, ctx->d_router_w, ctx->d_router_b,
+                  reinterpret_cast<const PageUpdate*>(ctx->d_pf_in + 1 + 4 * C + 2 * Smax), ctx->d_pf_in, st);
+    PrefillDev P{};
+    P.T = T;
+    P.S = S;
+    P.C = C;
+    P.Smax = Smax;
+    P.seqidx = ctx->d_pf_in + 1 + 2 * C;
+    P.pos = ctx->d_pf_in + 1 + 3 * C;
+    P.seq_slot = ctx->d_pf_in + 1 + 4 * C;
+    P.m = ctx->d_pf_m;
+    P.idx = ctx->d_pf_idx;
+    P.n = ctx->d_pf_n;
+    P.row_slot = ctx->d_pf_row_slot;
+    P.row_cslot = ctx->d_pf_row_cslot;
+    P.row_pos = ctx->d_pf_row_pos;
+    P.first = ctx->d_pf_first;
+    P.cnt = ctx->d_pf_cnt;
+    P.s0 = ctx->d_pf_s0;
+    P.tile_base = ctx->d_pf_tile_base;
+    P.len = ctx->d_len;
+    launch_pf_plan(md, P, st);
+    StepDev sp{};
+    sp.page_table = ctx->d_page_table;
+    sp.pool = ctx->d_pool;
+    sp.pos_table = ctx->d_pos_table;
+    sp.len = ctx->d_len;
+    sp.err = ctx->d_err;
+    for (int r = 0; r < M; ++r) {
+      const int* n_dev = ctx->d_pf_n + r;
+      const int* idx_r = ctx->d_pf_idx + (size_t)r * C;
+      for (int j = 0; j < J; ++j) {
+        launch_norm_rows(md.dtype, ctx->d_pf_H, md.d, idx_r, n_dev, 0, C, ctx->d_attn_norm + (size_t)j * md.d, md.d,
+                         md.eps, ctx->d_pf_X, md.d, st);
+        GemmArgs a{};
+        a.n_dev = n_dev;
+        a.epi = EPI_CL_QKV;
+        a.md = md;
+        a.s = sp;
+        a.r = r;
+        a.j = j;
+        a.inv_freq = ctx->d_inv_freq;
+        a.Q = ctx->d_pf_Q;
+        a.row_slot = ctx->d_pf_row_slot + (size_t)r * C;
+        a.row_cslot = ctx->d_pf_row_cslot + (size_t)r * C;
+        a.row_pos = ctx->d_pf_row_pos + (size_t)r * C;
+        gemm_pf(ctx, ctx->wqkv[j], &ctx->pf_map_X, a, st);
+        launch_pf_attn(md, P, sp, r, j, ctx->d_pf_Q, ctx->d_pf_O, C / 32 + S + 1, st);
+        a = GemmArgs{};
+        a.n_dev = n_dev;
+        a.epi = EPI_CL_RESID;
+        a.resid = ctx->d_pf_H;
+        a.ldr = md.d;
+        a.idx = idx_r;
+        gemm_pf(ctx, ctx->wo[j], &ctx->pf_map_O, a, st);
+        launch_norm_rows(md.dtype, ctx->d_pf_H, md.d, idx_r, n_dev, 0, C, ctx->d_mlp_norm + (size_t)j * md.d, md.d,
+                         md.eps, ctx->d_pf_X, md.d, st);
+        a = GemmArgs{};
+        a.n_dev = n_dev;
+        a.epi = EPI_CL_SWIGLU;
+        a.md = md;
+        a.U = ctx->d_pf_U;
+        gemm_pf(ctx, ctx->wgu[j], &ctx->pf_map_X, a, st);
+        a = GemmArgs{};
+        a.n_dev = n_dev;
+        a.epi = EPI_CL_RESID;
+        a.resid = ctx->d_pf_H;
+        a.ldr = md.d;
+        a.idx = idx_r;
+        gemm_pf(ctx, ctx->wd[j], &ctx->pf_map_U, a, st);
+      }
+    }
+    if (last_logits && nend > 0) {
+      for (int e0 = 0; e0 < nend; e0 += maxB) {
+        const int cnt = std::min(maxB, nend - e0);
+        launch_norm_rows(md.dtype, ctx->d_pf_H, md.d, ctx->d_pf_in + 1 + 4 * C + Smax + e0, nullptr, cnt, cnt,
+                         ctx->d_final_norm, md.d, md.eps, ctx->d_Xf, md.d, st);
+        GemmArgs a{};
+        a.n_host = cnt;
+        a.max_rows = maxB;
+        a.epi = EPI_STORE;
+        a.out = ctx->d_logits;
+        a.ldo = md.V;
+        a.splits = 1;
+        gemm(ctx, ctx->emb_mat, &ctx->map_Xf, ctx->d_Xf, md.d, a, st);
+        for (int e = 0; e < cnt; ++e)
+          CK(ctx, cudaMemcpyAsync(last_logits + (size_t)ending[e0 + e] * md.V, ctx->d_logits + (size_t)e * md.V,
+                                  (size_t)md.V * 4, logits_dev ? cudaMemcpyDeviceToDevice : cudaMemcpyDeviceToHost,
+                                  st));
+      }
+    }
+    launch_pf_len(md, P, st);
+    CK(ctx, cudaGetLastError());
+    CK(ctx, cudaMemcpyAsync(ctx->h_pf_m, ctx->d_pf_m, (size_t)T * 4, cudaMemcpyDeviceToHost, st));
+    CK(ctx, cudaMemcpyAsync(ctx->h_err, ctx->d_err, 4, cudaMemcpyDeviceToHost, st));
+    CK(ctx, cudaStreamSynchronize(st));
+    if (*ctx->h_err) {
+      const uint32_t e = *ctx->h_err;
+      cudaMemsetAsync(ctx->d_err, 0, 4, st);
+      return fail(ctx, TLF_ERR_DEVICE, "device error word 0x%x during prefill", e);
+    }
+    // loop counts out, host lengths, and the pages the worst-case reservation did not need
+    for (int si = 0, t = 0; si < S; ++si) {
+      const Seg& g = segs[si];
+      const int slot = slot_of[g.s];
+      for (int i = 0; i < g.count; ++i, ++t) {
+        const int m = ctx->h_pf_m[t];
+        if (loops) loops[offsets[g.s] + g.start + i] = m;
+        for (int r = 0; r < m; ++r) ctx->h_len[(size_t)slot * M + r] += 1;
+      }
+      for (int r = 0; r < M; ++r) {
+        const int keep = (ctx->h_len[(size_t)slot * M + r] + ps - 1) / ps;
+        for (int p = keep; p < md.max_pages; ++p) {
+          int& e = pt_at(ctx, slot, r, p);
+          if (e < 0) break;
+          ctx->free_pages.push_back(e);
+          e = -1;
+        }
+      }
+    }
+  }
+  return TLF_OK;
+}
+
 extern "C" int tlf_prefill(tlf_ctx* ctx, int32_t n_seqs, const uint64_t* seq_ids, const int32_t* offsets,
                            const int32_t* tokens, const int32_t* forced, float* last_logits, int32_t* loops,
                            void* stream) {
@@ -900,6 +1190,12 @@ extern "C" int tlf_prefill(tlf_ctx* ctx, int32_t n_seqs, const uint64_t* seq_ids
     return rc;
   };
   const bool logits_dev = last_logits && is_device_ptr(last_logits);
+  if (ctx->use_tc) {  // batched, chunked prefill on the tensor-core path
+    const int rc = prefill_batched(ctx, n_seqs, slot_of.data(), offsets, tokens, forced, last_logits, logits_dev,
+                                   loops, st);
+    return rc ? rollback(rc) : TLF_OK;
+  }
+  // float32 models: the prompt runs position by position through the decode kernels
   const int maxB = ctx->cfg.max_batch;
   std::vector<PageUpdate> upd;
   for (int g0 = 0; g0 < n_seqs; g0 += maxB) {

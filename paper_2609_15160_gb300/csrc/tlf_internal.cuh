@@ -351,6 +351,12 @@ struct GemmArgs {
   const double* inv_freq;  // [hd/2] rotary frequencies
   float* Q;                // [max_rows][Hq][hd]
   void* U;                 // [max_rows][ff] bf16
+  // token tiling (prefill): gridDim.z = tok_tiles tiles of NT rows
+  int tok_tiles;
+  // prefill QKV epilogue: per compact row, sequence slot, loop-r cache slot and position
+  const int* row_slot;
+  const int* row_cslot;
+  const int* row_pos;
 };
 
 // ----------------------------------------------------------------------------
@@ -389,6 +395,32 @@ void launch_scatter_cache(const ModelDims& md, int slot, int r, int n, const voi
                           cudaStream_t st);
 void launch_fill_cache(const ModelDims& md, int slot, int r, int n, const int* positions, const int* page_table,
                        void* pool, int* pos_table, cudaStream_t st);
+
+// Batched prefill of one chunk of prompt tokens (ordered by sequence, then position).
+struct PrefillDev {
+  int T;               // tokens in the chunk
+  int S;               // sequences in the chunk (<= Smax <= 1024)
+  int C;               // chunk capacity (row stride of the per-loop arrays)
+  int Smax;            // sequence capacity (row stride of the per-sequence arrays)
+  const int* seqidx;   // [T] sequence of each token (0..S-1)
+  const int* pos;      // [T] original position of each token
+  const int* seq_slot; // [S] sequence slot
+  const int* m;        // [T] loop counts
+  int* idx;            // [M][C] chunk rows of A_r
+  int* n;              // [M] |A_r|
+  int* row_slot;       // [M][C] sequence slot of each compact row
+  int* row_cslot;      // [M][C] loop-r cache slot of each compact row
+  int* row_pos;        // [M][C] position of each compact row
+  int* first;          // [M][Smax] first compact row of each sequence
+  int* cnt;            // [M][Smax] compact rows of each sequence
+  int* s0;             // [M][Smax] loop-r cache length of each sequence before the chunk
+  int* tile_base;      // [M][Smax + 1] attention query blocks, prefix over sequences
+  int* len;            // [max_seqs][M] cache lengths
+};
+void launch_pf_plan(const ModelDims& md, const PrefillDev& p, cudaStream_t st);
+void launch_pf_attn(const ModelDims& md, const PrefillDev& p, const StepDev& s, int r, int j, const float* Q,
+                    void* O, int tiles_bound, cudaStream_t st);
+void launch_pf_len(const ModelDims& md, const PrefillDev& p, cudaStream_t st);
 
 // Kernel-level attention operation (tlf_attn_decode): scratch layout and launch.
 struct AttnOpLayout {

@@ -32,7 +32,7 @@ class TlfConfig(C.Structure):
                                          "ffn_hidden", "max_loops")] + [
         ("rope_base", C.c_float), ("norm_eps", C.c_float), ("dtype", C.c_int32), ("exit_rule", C.c_int32),
         ("threshold", C.c_float), ("max_seqs", C.c_int32), ("max_batch", C.c_int32), ("max_seq_len", C.c_int32),
-        ("page_size", C.c_int32), ("gemm_impl", C.c_int32), ("host_only", C.c_int32), ("reserved0", C.c_int32),
+        ("page_size", C.c_int32), ("gemm_impl", C.c_int32), ("host_only", C.c_int32), ("prefill_chunk", C.c_int32),
         ("kv_pool_pages", C.c_int64)]
 
 
@@ -138,12 +138,13 @@ def _stream(stream) -> Optional[int]:
 # ----------------------------------------------------------------------------
 
 def make_config(m, max_seqs: int, max_batch: int, max_seq_len: int, page_size: int = 64,
-                kv_pool_pages: int = 0, gemm_impl: str = "auto", host_only: bool = False) -> TlfConfig:
+                kv_pool_pages: int = 0, gemm_impl: str = "auto", host_only: bool = False,
+                prefill_chunk: int = 0) -> TlfConfig:
     return TlfConfig(vocab=m.vocab, d_model=m.d_model, n_heads=m.n_heads, n_kv_heads=m.n_kv_heads,
                      head_dim=m.head_dim, n_layers=m.n_layers, ffn_hidden=m.ffn_hidden, max_loops=m.max_loops,
                      rope_base=m.rope_base, norm_eps=m.norm_eps, dtype=DTYPE[m.dtype], exit_rule=EXIT[m.exit_rule],
                      threshold=m.threshold, max_seqs=max_seqs, max_batch=max_batch, max_seq_len=max_seq_len,
-                     page_size=page_size, gemm_impl=GEMM[gemm_impl], host_only=int(host_only), reserved0=0,
+                     page_size=page_size, gemm_impl=GEMM[gemm_impl], host_only=int(host_only), prefill_chunk=prefill_chunk,
                      kv_pool_pages=kv_pool_pages)
 
 
@@ -242,10 +243,11 @@ class Context:
     """One library context for a model configuration (synth.ModelConfig)."""
 
     def __init__(self, model, weights: Optional[Dict[str, np.ndarray]], max_seqs: int, max_batch: int,
-                 max_seq_len: int, kv_pool_pages: int = 0, gemm_impl: str = "auto", host_only: bool = False):
+                 max_seq_len: int, kv_pool_pages: int = 0, gemm_impl: str = "auto", host_only: bool = False,
+                 prefill_chunk: int = 0):
         self.model = model
         self.cfg = make_config(model, max_seqs, max_batch, max_seq_len, kv_pool_pages=kv_pool_pages,
-                               gemm_impl=gemm_impl, host_only=host_only)
+                               gemm_impl=gemm_impl, host_only=host_only, prefill_chunk=prefill_chunk)
         self.handle, _ = tlf_create(self.cfg, weights, model.dtype)
         self.max_batch = max_batch
 

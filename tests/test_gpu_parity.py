@@ -274,6 +274,31 @@ def test_profile_counters(tlf):
         assert abs(by - want) < 1e-6 * want
 
 
+@pytest.mark.parametrize("lens", [[600, 5, 257], [300] * 3 + [1] * 70])
+def test_chunked_batched_prefill(tlf, lens):
+    """Prompts spanning several 256-token prefill chunks (and more sequences than one chunk holds)."""
+    m = _small(vocab=400, max_loops=3, depth_probs=(0.3, 0.3, 0.4))
+    w = synth.make_weights(m)
+    om = O.OracleModel.from_config(m, w)
+    depth = DepthOracle(om)
+    rng = np.random.default_rng(17)
+    prompts = [rng.integers(0, m.vocab, size=n).astype(np.int32) for n in lens]
+    ids = list(range(50, 50 + len(prompts)))
+    with tlf.Context(m, w, max_seqs=len(prompts), max_batch=min(64, len(prompts)), max_seq_len=700,
+                     prefill_chunk=256) as ctx:
+        pf = [depth.forced_for(p) for p in prompts]
+        glog, gl = ctx.prefill(ids, prompts, forced=pf)
+        for b in (0, 1, 2, len(prompts) - 1):
+            seq = O.OracleSequence(om)
+            olog, oml = O.prefill_gathered(om, seq, prompts[b], forced=pf[b])
+            np.testing.assert_array_equal(gl[b], oml)
+            assert rel_err(glog[b], olog) < tol_for(m)
+            check_cache(ctx, ids[b], seq, m)
+        live, free, total = ctx.stats()
+        used = sum(sum((ctx.cache_len(i, r) + 63) // 64 for r in range(1, m.max_loops + 1)) for i in ids)
+        assert total - free == used  # the worst-case reservation was trimmed
+
+
 def test_device_filled_restore(tlf):
     """tlf_load_cache without values: lengths and positions as given, values on the 1/64 grid in [-2, 2)."""
     m = _small()
