@@ -53,6 +53,17 @@ def _measured_peaks():
     return 6800.0, "fallback"
 
 
+def _attn_traffic(alg_bytes_per_launch: float):
+    """DRAM bytes per attention launch, scaled from the committed ncu capture (None if absent)."""
+    p = os.path.join(ROOT, "profiles", "traffic.json")
+    try:
+        with open(p) as f:
+            ratio = json.load(f)["k_attn_decode"]["traffic_over_algorithmic"]
+    except (OSError, KeyError, ValueError):
+        return None
+    return ratio * alg_bytes_per_launch
+
+
 class ClockSampler:
     """nvidia-smi clock / throttle samples during the timed region."""
 
@@ -329,7 +340,9 @@ def run_ours(args):
             "roofline": {"bound": "hbm", "kernel": "k_attn_decode (recursion-wise split-K attention)",
                          "achieved": att_gbs, "peak": peak, "unit": "GB/s",
                          "frac": (att_gbs / peak) if att_gbs else None, "peak_kind": peak_kind,
-                         "traffic": None,
+                         "traffic": _attn_traffic(att_bytes / max(1, att_launches)),
+                         "traffic_source": "ncu dram bytes / algorithmic bytes of one captured launch "
+                                           "(profiles/traffic.json) x this launch's algorithmic bytes",
                          "algorithmic_bytes_per_launch": att_bytes / max(1, att_launches),
                          "avg_launch_ms": att_ms / max(1, att_launches)},
             "e2e": {"value": ws * B * args.steps / (e2e_ms * 1e-3), "unit": "tokens/s",

@@ -35,29 +35,39 @@ __global__ void __launch_bounds__(256) k_router(ModelDims md, StepDev s, int B, 
     if (lane == 0) atomicOr(s.err, DEVERR_INDEX);
     tok = 0;
   }
+  // One pass over 16-byte chunks: each chunk of E[x] is loaded once, written to
+  // the residual stream, squared into the norm, and dotted with all M router rows;
+  // the RMSNorm scale (a per-row scalar) multiplies the dot products afterwards.
+  constexpr int VEC = Vec16<T>::N;
   const T* e = emb + (size_t)tok * d;
   float* h = s.H + (size_t)b * d;
-  float ss = 0.f;
-  for (int i = lane; i < d; i += 32) {
-    const float x = to_f32(e[i]);
-    h[i] = x;
-    ss += x * x;
+  float ss = 0.f, dot[16];
+#pragma unroll
+  for (int l = 0; l < 16; ++l) dot[l] = 0.f;
+  for (int c = lane; c < d / VEC; c += 32) {
+    float x[VEC];
+    Vec16<T>::load(e + c * VEC, x);
+#pragma unroll
+    for (int u = 0; u < VEC; u += 4)
+      *reinterpret_cast<float4*>(h + c * VEC + u) = make_float4(x[u], x[u + 1], x[u + 2], x[u + 3]);
+#pragma unroll
+    for (int u = 0; u < VEC; ++u) ss = fmaf(x[u], x[u], ss);
+#pragma unroll
+    for (int l = 0; l < 16; ++l) {
+      if (l < M) {
+        float w[VEC];
+        Vec16<T>::load(rw + (size_t)l * d + c * VEC, w);
+#pragma unroll
+        for (int u = 0; u < VEC; ++u) dot[l] = fmaf(x[u], w[u], dot[l]);
+      }
+    }
   }
   ss = warp_sum(ss);
   const float inv = rsqrtf(ss / (float)d + md.eps);
 
   float z[16];
 #pragma unroll
-  for (int l = 0; l < 16; ++l) {
-    if (l < M) {
-      const T* w = rw + (size_t)l * d;
-      float acc = 0.f;
-      for (int i = lane; i < d; i += 32) acc += (to_f32(e[i]) * inv) * to_f32(w[i]);
-      z[l] = warp_sum(acc) + rb[l];
-    } else {
-      z[l] = -INFINITY;
-    }
-  }
+  for (int l = 0; l < 16; ++l) z[l] = (l < M) ? warp_sum(dot[l]) * inv + rb[l] : -INFINITY;
 
   int m = 1;
   float margin;
