@@ -116,6 +116,22 @@ def _dist():
     return ws, rank, local
 
 
+def max_over_ranks(values, device="cpu"):
+    """Element-wise maximum of per-rank floats over the process group (identity without one)."""
+    import torch
+    import torch.distributed as dist
+
+    t = torch.tensor(values, dtype=torch.float64, device=device)
+    if dist.is_available() and dist.is_initialized() and dist.get_world_size() > 1:
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return t.tolist()
+
+
+def job_tokens_per_s(world_size: int, batch_per_rank: int, steps: int, slowest_ms: float) -> float:
+    """Whole-job decode throughput: the tokens of every rank over the slowest rank's time."""
+    return world_size * batch_per_rank * steps / (slowest_ms * 1e-3)
+
+
 def _oracle_sample_cmd(cfg_name: str, tokens: int, rank_seed: int) -> str:
     return f"""
 import sys, time, json, numpy as np
@@ -299,10 +315,7 @@ def run_ours(args):
             breakdown[kname] = breakdown.get(kname, 0.0) + kms / args.steps
     ctx.set_profiling(False)
 
-    times = torch.tensor([total_ms, e2e_ms], dtype=torch.float64, device="cuda")
-    if ws > 1:
-        torch.distributed.all_reduce(times, op=torch.distributed.ReduceOp.MAX)
-    total_ms, e2e_ms = times.tolist()
+    total_ms, e2e_ms = max_over_ranks([total_ms, e2e_ms], device="cuda")
     # algorithmic HBM bytes of the timed steps: the weights of every loop that had an active
     # token (read once per loop), the LM head, and the K/V every active token reads and writes
     eb = 2 if m.dtype == "bf16" else 4
@@ -318,7 +331,7 @@ def run_ours(args):
     if rank == 0:
         peak, peak_kind = _measured_peaks()
         att_gbs = att_bytes / (att_ms * 1e-3) / 1e9 if att_ms > 0 else None
-        value = ws * B * args.steps / (total_ms * 1e-3)
+        value = job_tokens_per_s(ws, B, args.steps, total_ms)
         h2d = B * 12
         d2h = B * m.vocab * 4 + B * 8
         line = {
@@ -345,7 +358,7 @@ def run_ours(args):
                                            "(profiles/traffic.json) x this launch's algorithmic bytes",
                          "algorithmic_bytes_per_launch": att_bytes / max(1, att_launches),
                          "avg_launch_ms": att_ms / max(1, att_launches)},
-            "e2e": {"value": ws * B * args.steps / (e2e_ms * 1e-3), "unit": "tokens/s",
+            "e2e": {"value": job_tokens_per_s(ws, B, args.steps, e2e_ms), "unit": "tokens/s",
                     "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h},
             "gpu_launches": int(launches),
             "kernel_ms_per_step_profiled": {k: round(v, 4) for k, v in breakdown.items()},
