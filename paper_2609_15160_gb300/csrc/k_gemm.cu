@@ -15,10 +15,20 @@
 // k_gemm_simt: CUDA-core tiled GEMM with the same epilogues, for float32
 // models (tcgen05 has no exact float32 mode) and as a second GPU path.
 //
-// Epilogues: split-K partial sums (consumed by RoPE/append and SwiGLU),
-// residual add + scatter into the float32 stream H[idx[row]] (Eq. 7, with
-// atomics so split-K partials need no extra pass), or a plain float32 store
-// (logits).
+// Epilogues of the bf16 decode path (cluster epilogues): the S split-K CTAs
+// of one 128-feature tile are launched as a (1, S, 1) thread-block cluster.
+// Each stages its partial tile in shared memory; after a cluster barrier
+// every CTA sums a 1/S share of the tile over the cluster through distributed
+// shared memory (fixed order, so results are deterministic) and finishes it:
+// residual add + scatter into the float32 stream H[idx[row]] (Eq. 7, one
+// writer per element), RoPE on q and k at the token's original position with
+// k and v appended to its loop-r page (Eq. 9, 11), or silu(gate) * up
+// (SwiGLU; gate and up rows interleave per 64-feature tile so one tile holds
+// both halves). No partial sum leaves the chip and no separate kernel runs.
+//
+// Other epilogues (SIMT path, prefill, LM head): split-K partial sums to a
+// buffer consumed by k_rope_append / k_swiglu, atomic residual add + scatter,
+// or a plain float32 store (logits).
 #include "tlf_internal.cuh"
 
 namespace tlf {
