@@ -49,17 +49,26 @@ __device__ __forceinline__ void gemm_write(const GemmArgs& a, int split, int row
 // ----------------------------------------------------------------------------
 constexpr int TC_BM = 128;
 constexpr int TC_BK = 64;  // 64 bf16 = one 128-byte swizzle row
-constexpr int TC_STAGES = 4;
+constexpr int TC_STAGES = 4;  // deepest operand ring; a launch uses min(4, k-tiles per CTA) stages
 
-template <int NT>
-constexpr int tc_smem_bytes() {
-  return 1024 /*align slack*/ + TC_STAGES * (TC_BM * TC_BK * 2 + NT * TC_BK * 2) + 256 /*barriers, tmem slot*/;
+// Dynamic shared memory of one CTA: the operand ring (reused after the main loop
+// for the cluster epilogue's fp32 partial tile [NT columns][128 features]), the
+// mbarriers and TMEM slot, and one int4 of per-column information per token.
+constexpr int tc_ring_bytes(int nt, int stages) { return stages * (TC_BM * TC_BK * 2 + nt * TC_BK * 2); }
+constexpr int tc_red_bytes(int nt) { return TC_BM * nt * 4; }
+constexpr int tc_body_bytes(int nt, int stages) {
+  return tc_ring_bytes(nt, stages) > tc_red_bytes(nt) ? tc_ring_bytes(nt, stages) : tc_red_bytes(nt);
+}
+constexpr int tc_smem_bytes(int nt, int stages) {
+  return 1024 /*align slack*/ + tc_body_bytes(nt, stages) + 256 /*barriers, tmem slot*/ + nt * 16;
 }
 
 // Second half of a cluster epilogue. Every CTA of the cluster has staged its
-// fp32 partial tile [128 features][NT + 1] at `red`; this CTA sums the partners'
-// tiles over its share of the token columns through distributed shared memory
-// and finishes them according to the mode.
+// fp32 partial tile [NT columns][128 features] at `red`; this CTA sums the
+// partners' tiles over its share of the token columns through distributed
+// shared memory and finishes them according to the mode. `ci[c]` holds what
+// the mode needs per token column c: the residual row (RESID, in .w), or the
+// page, slot in page and position of the token's new cache entry (QKV).
 constexpr int CL_MAX = 8;  // largest cluster (split-K factor) of the cluster epilogues
 
 // Sums over the cluster of the staged values at feature f, columns c..c+3
@@ -82,7 +91,7 @@ __device__ __forceinline__ void cluster_sum4(const uint32_t* pb, int S, int f, i
 }
 
 template <int NT>
-__device__ void cluster_epilogue(const GemmArgs& a, float* red, int* colinfo, int m0, int n, int tok0) {
+__device__ void cluster_epilogue(const GemmArgs& a, float* red, int4* ci, int m0, int n, int tok0) {
   const int S = a.splits;
   const int rank = (int)cluster_ctarank();
   const int per = (n + S - 1) / S;
@@ -101,10 +110,8 @@ __device__ void cluster_epilogue(const GemmArgs& a, float* red, int* colinfo, in
         cluster_sum4(pb, S, tid, c, c1, sm);
 #pragma unroll
         for (int q = 0; q < 4; ++q)
-          if (c + q < c1) {
-            const int row = a.idx ? a.idx[tok0 + c + q] : tok0 + c + q;
-            atomicAdd(a.resid + (size_t)row * a.ldr + col, sm[q]);  // the only writer of this element
-          }
+          if (c + q < c1)  // the only writer of this element
+            atomicAdd(a.resid + (size_t)ci[c + q].w * a.ldr + col, sm[q]);
       }
     return;
   }
@@ -123,47 +130,41 @@ __device__ void cluster_epilogue(const GemmArgs& a, float* red, int* colinfo, in
       }
     return;
   }
-  // EPI_CL_QKV: column c is token k = c of A_r
+  // EPI_CL_QKV: column c is token k = tok0 + c of A_r
   const ModelDims& md = a.md;
   const StepDev& s = a.s;
   const int ps = md.page_size, hd = md.hd, half = hd / 2;
-  int* ci_pos = colinfo;
-  int* ci_page = colinfo + NT;
-  int* ci_off = colinfo + 2 * NT;
-  for (int t = tid; t < c1 - c0; t += blockDim.x) {
-    const int row = tok0 + c0 + t;
-    int slot, L, pos;
-    if (a.row_cslot) {  // prefill: per-row sequence slot, cache slot and position from the plan
-      slot = a.row_slot[row];
-      L = a.row_cslot[row];
-      pos = a.row_pos[row];
-    } else {            // decode: the token appends at the end of its loop-r cache
-      slot = s.slots[s.idx[a.r * md.max_batch + row]];
-      L = s.len[slot * md.M + a.r];
-      pos = s.len[slot * md.M];  // every token runs loop 1: its length is the token count
+  if (a.row_cslot) {
+    // prefill: sequence slot, cache slot and position of each row from the prefill plan
+    for (int c = c0 + tid; c < c1; c += blockDim.x) {
+      const int row = tok0 + c;
+      const int slot = a.row_slot[row], L = a.row_cslot[row];
+      int pos = a.row_pos[row];
+      int page = s.page_table[((size_t)slot * md.M + a.r) * md.max_pages + L / ps];
+      if (page < 0 || page >= md.n_pages || pos < 0 || pos >= md.max_pos) {
+        atomicOr(s.err, DEVERR_INDEX);
+        page = -1;
+        pos = 0;
+      } else if (a.j == 0) {
+        s.pos_table[(size_t)page * ps + L % ps] = pos;
+      }
+      ci[c] = make_int4(page, L % ps, pos, 0);
     }
-    int page = s.page_table[((size_t)slot * md.M + a.r) * md.max_pages + L / ps];
-    if (page < 0 || page >= md.n_pages) {
-      atomicOr(s.err, DEVERR_INDEX);
-      page = -1;
-    }
-    ci_pos[t] = pos;
-    ci_page[t] = page;
-    ci_off[t] = L % ps;
-    if (a.j == 0 && page >= 0) s.pos_table[(size_t)page * ps + L % ps] = pos;
+    __syncthreads();
   }
-  __syncthreads();
   const int gfeat = m0 + tid;
   if (gfeat >= md.qkv_dim) return;
-  const double two_pi = 6.283185307179586476925286766559;
   bf16* pool = reinterpret_cast<bf16*>(s.pool);
   if (gfeat < md.q_dim + md.kv_dim) {
     const bool is_q = gfeat < md.q_dim;
     const int fr = is_q ? gfeat : gfeat - md.q_dim;
     const int h = fr / hd, i = fr % hd;
     if (i >= half) return;  // the lower lane of the rotary pair handles both
-    const double freq = a.inv_freq[i];
     for (int c = c0; c < c1; c += 4) {
+      float2 csn[4];
+#pragma unroll
+      for (int q = 0; q < 4; ++q)
+        csn[q] = (c + q < c1) ? a.rope[(size_t)ci[c + q].z * half + i] : make_float2(1.f, 0.f);
       float x0[4], x1[4];
       cluster_sum4(pb, S, tid, c, c1, x0);
       cluster_sum4(pb, S, tid + half, c, c1, x1);
@@ -171,20 +172,19 @@ __device__ void cluster_epilogue(const GemmArgs& a, float* red, int* colinfo, in
       for (int q = 0; q < 4; ++q) {
         const int cc = c + q;
         if (cc >= c1) break;
-        double ang = (double)ci_pos[cc - c0] * freq;
-        ang -= two_pi * rint(ang / two_pi);
-        float sn, cs;
-        sincosf((float)ang, &sn, &cs);
-        const float r0 = x0[q] * cs - x1[q] * sn, r1 = x0[q] * sn + x1[q] * cs;
+        const float r0 = x0[q] * csn[q].x - x1[q] * csn[q].y, r1 = x0[q] * csn[q].y + x1[q] * csn[q].x;
         if (is_q) {
           float* qo = a.Q + ((size_t)(tok0 + cc) * md.Hq + h) * hd;
           qo[i] = r0;
           qo[i + half] = r1;
-        } else if (ci_page[cc - c0] >= 0) {
-          bf16* kp = pool + (size_t)ci_page[cc - c0] * md.page_elems +
-                     ((size_t)(a.j * 2 + 0) * md.Hkv + h) * ps * hd + (size_t)ci_off[cc - c0] * hd;
-          kp[i] = __float2bfloat16_rn(r0);
-          kp[i + half] = __float2bfloat16_rn(r1);
+        } else {
+          const int4 e = ci[cc];
+          if (e.x >= 0) {
+            bf16* kp = pool + (size_t)e.x * md.page_elems + ((size_t)(a.j * 2 + 0) * md.Hkv + h) * ps * hd +
+                       (size_t)e.y * hd;
+            kp[i] = __float2bfloat16_rn(r0);
+            kp[i + half] = __float2bfloat16_rn(r1);
+          }
         }
       }
     }
@@ -197,9 +197,9 @@ __device__ void cluster_epilogue(const GemmArgs& a, float* red, int* colinfo, in
 #pragma unroll
       for (int q = 0; q < 4; ++q) {
         const int cc = c + q;
-        if (cc < c1 && ci_page[cc - c0] >= 0) {
-          bf16* vp = pool + (size_t)ci_page[cc - c0] * md.page_elems +
-                     ((size_t)(a.j * 2 + 1) * md.Hkv + h) * ps * hd + (size_t)ci_off[cc - c0] * hd;
+        if (cc < c1 && ci[cc].x >= 0) {
+          bf16* vp = pool + (size_t)ci[cc].x * md.page_elems + ((size_t)(a.j * 2 + 1) * md.Hkv + h) * ps * hd +
+                     (size_t)ci[cc].y * hd;
           vp[i] = __float2bfloat16_rn(x[q]);
         }
       }
@@ -215,10 +215,12 @@ __global__ void __launch_bounds__(128) k_gemm_tc(const __grid_constant__ CUtenso
   constexpr uint32_t TMEM_COLS = NT < 32 ? 32 : NT;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+  const int NS = a.stages;  // 1..TC_STAGES
   uint8_t* sA = smem;
-  uint8_t* sB = smem + TC_STAGES * A_BYTES;
-  uint64_t* bars = reinterpret_cast<uint64_t*>(sB + TC_STAGES * B_BYTES);
+  uint8_t* sB = smem + NS * A_BYTES;
+  uint64_t* bars = reinterpret_cast<uint64_t*>(smem + tc_body_bytes(NT, NS));
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 2 * TC_STAGES + 1);
+  int4* colinfo = reinterpret_cast<int4*>(reinterpret_cast<uint8_t*>(bars) + 256);  // [NT]
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   // The token count comes from the plan kernel, which completed before this
@@ -245,7 +247,7 @@ __global__ void __launch_bounds__(128) k_gemm_tc(const __grid_constant__ CUtenso
   const uint32_t done = smem_u32(&bars[2 * TC_STAGES]);
 
   if (threadIdx.x == 0) {
-    for (int i = 0; i < TC_STAGES; ++i) {
+    for (int i = 0; i < NS; ++i) {
       mbar_init(full(i), 1);
       mbar_init(empty(i), 1);
     }
@@ -266,7 +268,7 @@ __global__ void __launch_bounds__(128) k_gemm_tc(const __grid_constant__ CUtenso
   if (warp == 0 && lane == 0) {
     // TMA producer. Weight tiles of the first stages go out before the wait on
     // the preceding kernels (weights are never written by them); token tiles after.
-    const int pre = nk < TC_STAGES ? nk : TC_STAGES;
+    const int pre = nk < NS ? nk : NS;
     for (int i = 0; i < pre; ++i) {
       mbar_arrive_expect_tx(full(i), A_BYTES + B_BYTES);
       tma_load_2d(smem_u32(sA + i * A_BYTES), &mapW, (kb0 + i) * TC_BK, m0, full(i));
@@ -275,8 +277,8 @@ __global__ void __launch_bounds__(128) k_gemm_tc(const __grid_constant__ CUtenso
     pdl_trigger();
     for (int i = 0; i < pre; ++i) tma_load_2d(smem_u32(sB + i * B_BYTES), &mapX, (kb0 + i) * TC_BK, tok0, full(i));
     for (int i = pre; i < nk; ++i) {
-      const int st = i % TC_STAGES;
-      const uint32_t ph = (uint32_t)(i / TC_STAGES) & 1u;
+      const int st = i % NS;
+      const uint32_t ph = (uint32_t)(i / NS) & 1u;
       if (!mbar_wait(empty(st), ph ^ 1u, a.err)) break;
       mbar_arrive_expect_tx(full(st), A_BYTES + B_BYTES);
       const int kx = (kb0 + i) * TC_BK;
@@ -286,14 +288,25 @@ __global__ void __launch_bounds__(128) k_gemm_tc(const __grid_constant__ CUtenso
   } else {
     pdl_wait();
     pdl_trigger();
+    if (warp >= 2) {
+      // idle during the main loop: fetch what the epilogue needs per token column
+      // (outputs of the plan kernel, read after the wait)
+      for (int c = threadIdx.x - 64; c < n; c += 64) {
+        if (a.epi == EPI_CL_QKV && !a.row_cslot) {
+          colinfo[c] = a.s.rowinfo[a.r * a.md.max_batch + tok0 + c];
+        } else if (a.epi == EPI_CL_RESID) {
+          colinfo[c] = make_int4(0, 0, 0, a.idx ? a.idx[tok0 + c] : tok0 + c);
+        }
+      }
+    }
   }
   if (nk > 0) {
     if (warp == 1 && lane == 0) {
       // MMA issuer
       const uint32_t idesc = idesc_bf16_f32(TC_BM, ncols);
       for (int i = 0; i < nk; ++i) {
-        const int st = i % TC_STAGES;
-        const uint32_t ph = (uint32_t)(i / TC_STAGES) & 1u;
+        const int st = i % NS;
+        const uint32_t ph = (uint32_t)(i / NS) & 1u;
         if (!mbar_wait(full(st), ph, a.err)) break;
         tc_fence_after();
         const uint64_t da = smem_desc_sw128(smem_u32(sA + st * A_BYTES));
@@ -318,7 +331,6 @@ __global__ void __launch_bounds__(128) k_gemm_tc(const __grid_constant__ CUtenso
     // then reduce across the cluster. Every CTA reaches both cluster barriers.
     // tile layout [column][128 features]: a warp's partner reads are 128 contiguous bytes
     float* red = reinterpret_cast<float*>(smem);
-    int* colinfo = reinterpret_cast<int*>(red + 128 * NT);
     const int f = warp * 32 + lane;
     for (int c0 = 0; c0 < ncols; c0 += 16) {
       float v[16];
@@ -364,14 +376,34 @@ __global__ void __launch_bounds__(128) k_gemm_tc(const __grid_constant__ CUtenso
 
 int gemm_tc_max_nt() { return 256; }
 
+int gemm_tc_stages(int K, int splits) {
+  const int nkb = (K + TC_BK - 1) / TC_BK;
+  const int per_cta = (nkb + splits - 1) / splits;
+  return per_cta < 1 ? 1 : (per_cta > TC_STAGES ? TC_STAGES : per_cta);
+}
+
+int gemm_tc_smem_bytes(int nt, int stages) { return tc_smem_bytes(nt, stages); }
+
+// Every CTA allocates max(32, NT) TMEM columns and tcgen05.alloc blocks until
+// columns are free, so as many CTAs as shared memory lets share an SM (the
+// smallest ring, of any kernel instance with the same NT) must fit in its 512
+// columns; otherwise clusters waiting for partners could wait on each other.
+constexpr int SM_SMEM = 232448;  // shared memory per SM available to CTAs (227 KB + 1 KB per CTA)
+constexpr bool tmem_fits(int nt) {
+  return (SM_SMEM / (tc_smem_bytes(nt, 1) + 1024)) * (nt < 32 ? 32 : nt) <= 512;
+}
+static_assert(tmem_fits(16) && tmem_fits(32) && tmem_fits(64) && tmem_fits(128) && tmem_fits(256),
+              "co-resident CTAs would oversubscribe TMEM");
+
 template <int NT>
-static void launch_tc_nt(const CUtensorMap* mapW, const CUtensorMap* mapX, const GemmArgs& a, cudaStream_t st) {
+static void launch_tc_nt(const CUtensorMap* mapW, const CUtensorMap* mapX, GemmArgs a, cudaStream_t st) {
   static bool attr_set = false;
-  constexpr int smem = tc_smem_bytes<NT>();
   if (!attr_set) {
-    cudaFuncSetAttribute(k_gemm_tc<NT>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+    cudaFuncSetAttribute(k_gemm_tc<NT>, cudaFuncAttributeMaxDynamicSharedMemorySize, tc_smem_bytes(NT, TC_STAGES));
     attr_set = true;
   }
+  a.stages = gemm_tc_stages(a.K, a.splits);
+  const int smem = tc_smem_bytes(NT, a.stages);
   dim3 grid((a.N + TC_BM - 1) / TC_BM, a.splits, a.tok_tiles > 0 ? a.tok_tiles : 1);
   if (a.epi < EPI_CL_RESID) {
     launch_k(k_gemm_tc<NT>, grid, 128, smem, st, *mapW, *mapX, a);

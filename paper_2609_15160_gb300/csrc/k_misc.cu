@@ -2,6 +2,7 @@
 //
 // k_norm_rows    gather + RMSNorm: X[k] = RMSNorm(H[idx[k]]) * gain for the
 //                rows of the active set (Eq. 6 followed by the pre-norm).
+// k_rope_table   (cos, sin) of every position x rotary frequency, built once.
 // k_rope_append  sums the split-K partials of the fused QKV projection (Eq. 9),
 //                rotates q and k at the token's original position, keeps q for
 //                the attention kernel and appends k, v to the token's slot of
@@ -77,10 +78,29 @@ void launch_norm_rows(int dtype, const float* H, int ldh, const int* idx, const 
     launch_k(k_norm_rows<float>, rows_max, 256, 0, st, H, ldh, idx, n_dev, n_host, gain, d, eps, (float*)X, ldx);
 }
 
+// Rotary table: table[p][i] = (cos, sin)(p * theta_i), the angle formed and
+// reduced in float64 and rounded once to float32 (Eq. 11 positions, R4 reading).
+__global__ void k_rope_table(int max_pos, int half, const double* __restrict__ inv_freq, float2* __restrict__ table) {
+  const double two_pi = 6.283185307179586476925286766559;
+  const size_t n = (size_t)max_pos * half;
+  for (size_t e = blockIdx.x * (size_t)blockDim.x + threadIdx.x; e < n; e += (size_t)gridDim.x * blockDim.x) {
+    const int p = (int)(e / half), i = (int)(e % half);
+    double ang = (double)p * inv_freq[i];
+    ang -= two_pi * rint(ang / two_pi);
+    double sn, cs;
+    sincos(ang, &sn, &cs);
+    table[e] = make_float2((float)cs, (float)sn);
+  }
+}
+
+void launch_rope_table(const ModelDims& md, const double* inv_freq, float2* table, cudaStream_t st) {
+  k_rope_table<<<1024, 256, 0, st>>>(md.max_pos, md.hd / 2, inv_freq, table);
+}
+
 template <typename T>
 __global__ void __launch_bounds__(256) k_rope_append(ModelDims md, StepDev s, int r, int j,
                                                      const float* __restrict__ part, int splits, float* __restrict__ Q,
-                                                     const double* __restrict__ inv_freq) {
+                                                     const float2* __restrict__ rope) {
   pdl_wait();
   pdl_trigger();
   const int k = blockIdx.x;
@@ -89,21 +109,14 @@ __global__ void __launch_bounds__(256) k_rope_append(ModelDims md, StepDev s, in
   const int n_pairs = (md.Hq + md.Hkv) * hd2;   // rotated q and k pairs, then v elements
   const int t = blockIdx.y * blockDim.x + threadIdx.x;
   if (t >= n_pairs + md.Hkv * md.hd) return;
-  const int b = s.idx[r * md.max_batch + k];
-  const int slot = s.slots[b];
-  const int pos = s.len[slot * md.M + 0];  // every token runs loop 1: its length is the token count
-  const int L = s.len[slot * md.M + r];
+  // page, slot and position of the token's new loop-r entry, from the plan kernel
+  const int4 ri = s.rowinfo[r * md.max_batch + k];
+  const int page = ri.x, off = ri.y, pos = ri.z;
+  if (page < 0) return;
   const int ps = md.page_size, hd = md.hd, half = hd / 2;
-  const int page = s.page_table[((size_t)slot * md.M + r) * md.max_pages + L / ps];
-  if (page < 0 || page >= md.n_pages) {
-    if (t == 0) atomicOr(s.err, DEVERR_INDEX);
-    return;
-  }
-  const int off = L % ps;
   T* pg = reinterpret_cast<T*>(s.pool) + (size_t)page * md.page_elems;
   const size_t pstride = (size_t)md.max_batch * md.qkv_dim;
   const float* prow = part + (size_t)k * md.qkv_dim;
-  const double two_pi = 6.283185307179586476925286766559;
 
   if (t < n_pairs) {
     // q heads then k heads: rotate pair (i, i + hd/2) by pos * theta_i
@@ -114,11 +127,8 @@ __global__ void __launch_bounds__(256) k_rope_append(ModelDims md, StepDev s, in
       a += prow[sp * pstride + c0];
       c += prow[sp * pstride + c1];
     }
-    double ang = (double)pos * inv_freq[i];
-    ang -= two_pi * rint(ang / two_pi);
-    float sn, cs;
-    sincosf((float)ang, &sn, &cs);
-    const float ra = a * cs - c * sn, rc = a * sn + c * cs;
+    const float2 csn = rope[(size_t)pos * half + i];
+    const float ra = a * csn.x - c * csn.y, rc = a * csn.y + c * csn.x;
     if (h < md.Hq) {
       float* qo = Q + ((size_t)k * md.Hq + h) * hd;
       qo[i] = ra;
@@ -137,17 +147,16 @@ __global__ void __launch_bounds__(256) k_rope_append(ModelDims md, StepDev s, in
     T* vp = pg + ((size_t)(j * 2 + 1) * md.Hkv + h) * ps * hd + (size_t)off * hd;
     vp[e] = from_f32<T>(a);
   }
-  if (j == 0 && t == 0) s.pos_table[(size_t)page * ps + off] = pos;
 }
 
 void launch_rope_append(const ModelDims& md, const StepDev& s, int r, int j, const float* part, int splits, float* Q,
-                        const double* inv_freq, cudaStream_t st) {
+                        const float2* rope, cudaStream_t st) {
   const int work = (md.Hq + md.Hkv) * (md.hd / 2) + md.Hkv * md.hd;
   dim3 grid(md.max_batch, (work + 127) / 128);
   if (md.dtype == 1)
-    launch_k(k_rope_append<bf16>, grid, 128, 0, st, md, s, r, j, part, splits, Q, inv_freq);
+    launch_k(k_rope_append<bf16>, grid, 128, 0, st, md, s, r, j, part, splits, Q, rope);
   else
-    launch_k(k_rope_append<float>, grid, 128, 0, st, md, s, r, j, part, splits, Q, inv_freq);
+    launch_k(k_rope_append<float>, grid, 128, 0, st, md, s, r, j, part, splits, Q, rope);
 }
 
 template <typename T>

@@ -7,10 +7,12 @@
 // The same kernel applies the page-table updates the host queued for the step.
 //
 // k_plan: one CTA. For every loop r it builds A_r = {b : m_b >= r} in
-// increasing b with a warp ballot plus a block prefix scan, and the work plan
-// of the decode attention over the loop-r caches: the pages of every (token,
-// kv head) item, from the device-side cache lengths, laid out in one flat
-// order (prefix sums), which the attention grid splits evenly.
+// increasing b with a warp ballot plus a block prefix scan, the page, slot
+// and position of each active token's new loop-r cache entry (read by the
+// QKV epilogue that appends k, v), and the work plan of the decode attention
+// over the loop-r caches: the pages of every (token, kv head) item, from the
+// device-side cache lengths, laid out in one flat order (prefix sums), which
+// the attention grid splits evenly.
 #include "tlf_internal.cuh"
 
 namespace tlf {
@@ -177,6 +179,22 @@ __global__ void __launch_bounds__(256) k_plan(ModelDims md, StepDev s, int B) {
     if (active) {
       s.item_base[r * (maxB + 1) + k] = base;
       s.nch[r * maxB + k] = np;
+    }
+    if (active && s.rowinfo) {  // NULL for callers that only attend (no append this step)
+      // where the token's k, v go (Eq. 11): slot L - 1 of the loop-r cache, at its original
+      // position (its loop-1 length, since every token runs loop 1); the position table of the
+      // page is filled here once for all layers
+      const int e = L - 1;
+      int pos = s.len[slot * M];
+      int page = s.page_table[((size_t)slot * M + r) * md.max_pages + e / ps];
+      if (page < 0 || page >= md.n_pages || pos >= md.max_pos) {
+        atomicOr(s.err, DEVERR_INDEX);
+        page = -1;
+        pos = 0;
+      } else {
+        s.pos_table[(size_t)page * ps + e % ps] = pos;
+      }
+      s.rowinfo[r * maxB + k] = make_int4(page, e % ps, pos, 0);
     }
     if (b == 0) {
       s.n[r] = n_r;

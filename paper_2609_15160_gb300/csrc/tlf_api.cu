@@ -63,6 +63,8 @@ struct tlf_ctx {
   float* d_mlp_norm = nullptr;
   float* d_final_norm = nullptr;
   double* d_inv_freq = nullptr;
+  float2* d_rope = nullptr;     // [max_pos][hd/2] (cos, sin)
+  int4* d_rowinfo = nullptr;    // [M][max_batch]
   std::vector<DeviceMat> wqkv, wo, wgu, wd;
   DeviceMat emb_mat;
 
@@ -325,6 +327,7 @@ static int create_impl(tlf_ctx* ctx, const tlf_weights* w) {
   md.max_seqs = c.max_seqs; md.max_batch = c.max_batch; md.max_pages = max_pages_of(c); md.page_size = c.page_size;
   md.eps = c.norm_eps; md.rope_base = c.rope_base; md.threshold = c.threshold; md.exit_rule = c.exit_rule;
   md.dtype = c.dtype;
+  md.max_pos = c.max_seq_len;
   ctx->eb = c.dtype == TLF_DTYPE_BF16 ? 2 : 4;
   md.page_elems = (long long)md.J * 2 * md.Hkv * md.page_size * md.hd;
   ctx->n_pages = c.kv_pool_pages > 0 ? c.kv_pool_pages : (int64_t)c.max_seqs * c.max_loops * md.max_pages;
@@ -407,6 +410,11 @@ static int create_impl(tlf_ctx* ctx, const tlf_weights* w) {
     std::vector<double> inv(md.hd / 2);
     for (int i = 0; i < md.hd / 2; ++i) inv[i] = std::pow((double)c.rope_base, -2.0 * i / md.hd);
     if ((rc = upload(ctx, (void**)&ctx->d_inv_freq, inv.data(), inv.size() * sizeof(double), "inv_freq"))) return rc;
+    if ((rc = dev_alloc(ctx, &ctx->d_rope, (size_t)md.max_pos * (md.hd / 2) * sizeof(float2), "rotary table")))
+      return rc;
+    launch_rope_table(md, ctx->d_inv_freq, ctx->d_rope, 0);
+    CK(ctx, cudaGetLastError());
+    CK(ctx, cudaStreamSynchronize(0));
   }
 
   // KV pool and tables
@@ -439,15 +447,23 @@ static int create_impl(tlf_ctx* ctx, const tlf_weights* w) {
         !make_map(&ctx->map_Xf, ctx->d_Xf, B, d, d, ctx->nt_max))
       return fail(ctx, TLF_ERR_CUDA, "cuTensorMapEncodeTiled failed for an activation buffer");
   }
-  // split-K factors: enough CTAs to cover the SMs (2 per SM when the tile is small)
+  // split-K factors. tcgen05 path: the largest cluster size (<= 8, the portable
+  // limit) whose grid still fits in one wave, counting how many CTAs of the
+  // resulting ring depth share an SM (10 % margin for cluster placement).
   if (ctx->use_tc) {
-    // the splits of a tile form one thread-block cluster (at most 8 CTAs, the portable size)
-    const int per_sm = ctx->nt_max <= 64 ? 2 : 1;
-    const int target = per_sm * ctx->num_sms;
-    ctx->s_qkv = choose_splits((md.qkv_dim + 127) / 128, (d + 63) / 64, target, 8);
-    ctx->s_o = choose_splits((d + 127) / 128, (md.q_dim + 63) / 64, target, 8);
-    ctx->s_gu = choose_splits(ctx->wgu[0].N / 128, (d + 63) / 64, target, 8);
-    ctx->s_d = choose_splits((d + 127) / 128, (ff + 63) / 64, target, 8);
+    auto pick = [&](int tiles, int K) {
+      const int nkb = (K + 63) / 64;
+      for (int S = std::min(8, nkb); S > 1; --S) {
+        const int bytes = gemm_tc_smem_bytes(ctx->nt_max, gemm_tc_stages(K, S));
+        const int per_sm = std::min(16, 232448 / (bytes + 1024));
+        if (10LL * tiles * S <= 9LL * per_sm * ctx->num_sms) return S;
+      }
+      return 1;
+    };
+    ctx->s_qkv = pick((md.qkv_dim + 127) / 128, d);
+    ctx->s_o = pick((d + 127) / 128, md.q_dim);
+    ctx->s_gu = pick(ctx->wgu[0].N / 128, d);
+    ctx->s_d = pick((d + 127) / 128, ff);
   } else {
     const int target = 2 * ctx->num_sms;
     ctx->s_qkv = choose_splits((md.qkv_dim + 63) / 64, (d + 31) / 32, target, ctx->split_cap);
@@ -467,6 +483,7 @@ static int create_impl(tlf_ctx* ctx, const tlf_weights* w) {
   if ((rc = dev_alloc(ctx, &ctx->d_attn_part, attn_partial_floats(md, ctx->attn_grid) * 4, "attention partials")))
     return rc;
   if ((rc = dev_alloc(ctx, &ctx->d_attn_cnt, (size_t)B * md.Hkv * 4, "attention tickets"))) return rc;
+  if ((rc = dev_alloc(ctx, &ctx->d_rowinfo, (size_t)M * B * sizeof(int4), "row info"))) return rc;
   CK(ctx, cudaMemset(ctx->d_attn_cnt, 0, (size_t)B * md.Hkv * 4));
   if ((rc = dev_alloc(ctx, &ctx->d_logits, (size_t)B * V * 4, "logits"))) return rc;
   if ((rc = dev_alloc(ctx, &ctx->d_err, 16, "error word"))) return rc;
@@ -491,7 +508,7 @@ extern "C" void tlf_destroy(tlf_ctx* ctx) {
     cudaDeviceSynchronize();
     auto f = [](void* p) { if (p) cudaFree(p); };
     f(ctx->d_emb); f(ctx->d_router_w); f(ctx->d_router_b); f(ctx->d_attn_norm); f(ctx->d_mlp_norm);
-    f(ctx->d_final_norm); f(ctx->d_inv_freq);
+    f(ctx->d_final_norm); f(ctx->d_inv_freq); f(ctx->d_rope); f(ctx->d_rowinfo);
     for (auto* v : {&ctx->wqkv, &ctx->wo, &ctx->wgu, &ctx->wd})
       for (auto& m : *v) f(m.ptr);
     f(ctx->d_pool); f(ctx->d_pos_table); f(ctx->d_page_table); f(ctx->d_len); f(ctx->d_upload);
@@ -651,6 +668,7 @@ static int enqueue_step(tlf_ctx* ctx, int B, bool need_logits, bool prof, cudaSt
   s.pool = ctx->d_pool;
   s.err = ctx->d_err;
   s.cnt = ctx->d_attn_cnt;
+  s.rowinfo = ctx->d_rowinfo;
   const PageUpdate* d_upd = reinterpret_cast<const PageUpdate*>(ctx->d_upload + 1 + 3 * B);
 
   ctx->last_launches = 0;
@@ -686,7 +704,7 @@ static int enqueue_step(tlf_ctx* ctx, int B, bool need_logits, bool prof, cudaSt
         a.s = s;
         a.r = r;
         a.j = j;
-        a.inv_freq = ctx->d_inv_freq;
+        a.rope = ctx->d_rope;
         a.Q = ctx->d_Q;
         gemm(ctx, ctx->wqkv[j], &ctx->map_X, ctx->d_X, md.d, a, st);
         mark(3);
@@ -695,7 +713,7 @@ static int enqueue_step(tlf_ctx* ctx, int B, bool need_logits, bool prof, cudaSt
         a.out = ctx->d_part;
         gemm(ctx, ctx->wqkv[j], &ctx->map_X, ctx->d_X, md.d, a, st);
         mark(3);
-        launch_rope_append(md, s, r, j, ctx->d_part, ctx->s_qkv, ctx->d_Q, ctx->d_inv_freq, st);
+        launch_rope_append(md, s, r, j, ctx->d_part, ctx->s_qkv, ctx->d_Q, ctx->d_rope, st);
         ++ctx->last_launches;
         mark(4);
       }
@@ -1074,7 +1092,7 @@ static int prefill_batched(tlf_ctx* ctx, int n_seqs, const int* slot_of, const i
         a.s = sp;
         a.r = r;
         a.j = j;
-        a.inv_freq = ctx->d_inv_freq;
+        a.rope = ctx->d_rope;
         a.Q = ctx->d_pf_Q;
         a.row_slot = ctx->d_pf_row_slot + (size_t)r * C;
         a.row_cslot = ctx->d_pf_row_cslot + (size_t)r * C;

@@ -311,6 +311,9 @@ struct StepDev {
   int* nch;            // [M][maxB] chunks per token
   int* chunk;          // [M] keys per page
   int* cnt;            // [maxB * Hkv] attention merge tickets (zeroed by the plan kernel)
+  int4* rowinfo;       // [M][maxB] per compact row k of A_r: {page, slot in page, position, 0} of the
+                       // token's new loop-r cache entry (page -1 if the page table is corrupt);
+                       // NULL for callers that only attend (the plan then writes no append targets)
   // cache state
   int* len;            // [max_seqs][M] entries per (sequence, loop)
   int* page_table;     // [max_seqs][M][max_pages]
@@ -328,12 +331,14 @@ struct ModelDims {
   float eps, rope_base, threshold;
   int exit_rule;
   int dtype;             // 0 f32, 1 bf16
+  int max_pos;           // positions 0..max_pos-1 have a row in the rotary table
 };
 
 struct GemmArgs {
   int N;             // output features (rows of W)
   int K;             // reduction length
   int splits;        // split-K factor (gridDim.y; the cluster size for EPI_CL_*)
+  int stages;        // depth of the tcgen05 kernel's operand ring (set by the launcher)
   const int* n_dev;  // token rows n (device scalar), or NULL to use n_host
   int n_host;
   int epi;           // GemmEpilogue
@@ -348,7 +353,7 @@ struct GemmArgs {
   ModelDims md;
   StepDev s;
   int r, j;
-  const double* inv_freq;  // [hd/2] rotary frequencies
+  const float2* rope;      // [max_pos][hd/2] (cos, sin) of position x rotary frequency
   float* Q;                // [max_rows][Hq][hd]
   void* U;                 // [max_rows][ff] bf16
   // token tiling (prefill): gridDim.z = tok_tiles tiles of NT rows
@@ -378,9 +383,14 @@ void launch_gemm_simt(int dtype, const void* W, const void* X, int ldx, const Ge
 void launch_gemm_tc(const CUtensorMap* mapW, const CUtensorMap* mapX, int nt_max, const GemmArgs& a,
                     cudaStream_t st);
 int gemm_tc_max_nt();
+// operand-ring depth of a tcgen05 GEMM whose CTAs each reduce ceil(ceil(K/64)/splits) k-tiles,
+// and the dynamic shared memory one CTA of token tile nt then needs
+int gemm_tc_stages(int K, int splits);
+int gemm_tc_smem_bytes(int nt, int stages);
 
+void launch_rope_table(const ModelDims& md, const double* inv_freq, float2* table, cudaStream_t st);
 void launch_rope_append(const ModelDims& md, const StepDev& s, int r, int j, const float* part, int splits,
-                        float* Q, const double* inv_freq, cudaStream_t st);
+                        float* Q, const float2* rope, cudaStream_t st);
 void launch_attn_decode(const ModelDims& md, const StepDev& s, int r, int j, const float* Q, float* part, void* O,
                         int* cnt, int grid, cudaStream_t st);
 int attn_decode_grid(const ModelDims& md, int num_sms);
