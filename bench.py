@@ -195,7 +195,7 @@ def run_reference(args):
     print(json.dumps(line))
 
 
-def setup_workload(T, wl, rank: int, gemm_impl="auto", prefill="auto", extra_tokens: int = 0):
+def setup_workload(T, wl, rank: int, gemm_impl="auto", prefill="auto", extra_tokens: int = 0, ablation="none"):
     m = wl.model
     w = synth.make_weights(m)
     B = wl.batch
@@ -223,7 +223,7 @@ def setup_workload(T, wl, rank: int, gemm_impl="auto", prefill="auto", extra_tok
         snaps = None
         pages = B * m.max_loops * ((max(lengths) + steps_cap) // 64 + 2)
     ctx = T.Context(m, w, max_seqs=B, max_batch=B, max_seq_len=max(lengths) + steps_cap, kv_pool_pages=pages,
-                    gemm_impl=gemm_impl)
+                    gemm_impl=gemm_impl, ablation=ablation)
     if snaps is not None:
         for b in range(B):
             ctx.load_cache(ids[b], snaps[b])
@@ -260,7 +260,7 @@ def run_ours(args):
     B = wl.batch
     t0 = time.time()
     ctx, ids, how = setup_workload(T, wl, rank, prefill=args.prefill,
-                                   extra_tokens=3 * (args.warmup + args.steps))
+                                   extra_tokens=3 * (args.warmup + args.steps), ablation=args.ablation)
     setup_s = time.time() - t0
     stream = torch.cuda.current_stream()
     n_steps = args.warmup + args.steps
@@ -343,7 +343,8 @@ def run_ours(args):
             "config": {"workload": DESCR[args.config], "name": args.config, "batch_per_gpu": B,
                        "context": int(wl.prompt_len[1]), "cache": how,
                        "l2": "inputs larger than L2 (KV cache and weights stream from HBM every step)",
-                       "parallelism": f"replicas x{ws} (independent sequences per GPU)"},
+                       "parallelism": f"replicas x{ws} (independent sequences per GPU)",
+                       "ablation": args.ablation},
             "mean_loops": float(loops_seen.mean()),
             "step_roofline": {"bound": "hbm", "algorithmic_bytes_per_step": alg_bytes,
                               "floor_ms": alg_bytes / (peak * 1e9) * 1e3,
@@ -499,6 +500,8 @@ def main():
     ap.add_argument("--prefill", default="auto", choices=["auto", "snapshot", "real"])
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--decode-batch", type=int, default=0, help="override the workload's batch (C5 sweep)")
+    ap.add_argument("--ablation", default="none", choices=["none", "no_gather"],
+                    help="decode without the gather of Eq. 6 (all rows every loop, exited rows masked)")
     args = ap.parse_args()
     if args.warmup < 3:
         args.warmup = 3

@@ -73,6 +73,16 @@ enum tlf_exit_rule { TLF_EXIT_ARGMAX = 0, TLF_EXIT_SURVIVAL = 1 };
  * also used by tests as a second GPU path). */
 enum tlf_gemm_impl { TLF_GEMM_AUTO = 0, TLF_GEMM_SIMT = 1 };
 
+/* Ablations of the decode step (Sec. 4 ablation study, gather-scatter and
+ * recursion-wise KV cache). Each computes the same logits and loop counts as
+ * TLF_ABLATION_NONE and differs only in the work it does:
+ *   NO_GATHER  every loop r that has an active token runs the shared block on
+ *              all B rows of the step; rows with m <= r are masked: their
+ *              residual stream is not updated and they append nothing, but
+ *              their projections and attention over their loop-r caches run
+ *              (the cost of computing without the gather of Eq. 6). */
+enum tlf_ablation { TLF_ABLATION_NONE = 0, TLF_ABLATION_NO_GATHER = 1 };
+
 typedef struct tlf_config {
   int32_t vocab;        /* V; the LM head is tied to the embedding */
   int32_t d_model;      /* d, multiple of 64 */
@@ -95,6 +105,8 @@ typedef struct tlf_config {
   int32_t host_only;    /* 1: allocate nothing on a GPU; only validation and bookkeeping run */
   int32_t prefill_chunk;/* prompt tokens per batched-prefill chunk (bf16 models); 0 = 8192 */
   int64_t kv_pool_pages;/* pages in the KV pool; 0 = max_seqs * max_loops * ceil(max_seq_len / page_size) */
+  int32_t ablation;     /* tlf_ablation; 0 = the method as published */
+  int32_t reserved;     /* must be 0 */
 } tlf_config;
 
 /* Host pointers to the weights. Shapes use V, d, Hq, Hkv, hd, J, ff, M from

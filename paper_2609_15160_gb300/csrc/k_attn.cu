@@ -77,7 +77,8 @@ __global__ void __launch_bounds__(ATT_THREADS) k_attn_decode(ModelDims md, StepD
   const int maxB = md.max_batch, M = md.M, Hkv = md.Hkv;
   const int n_r = s.n[r];
   const int* pbase = s.item_base + r * (maxB + 1);  // first flat page of each token's items
-  const int* npg = s.nch + r * maxB;                 // pages of each of the token's items
+  const int* nkeys = s.nch + r * maxB;               // keys of each of the token's items (plan kernel)
+  auto pages_of = [&](int kk) { return (nkeys[kk] + ATT_PS - 1) / ATT_PS; };
   const int total = (n_r > 0) ? pbase[n_r] : 0;
   const int per = (total + gridDim.x - 1) / gridDim.x;
   const int p0 = blockIdx.x * per;
@@ -103,7 +104,7 @@ __global__ void __launch_bounds__(ATT_THREADS) k_attn_decode(ModelDims md, StepD
       if (pbase[mid] <= p) lo = mid; else hi = mid;
     }
     k = lo;
-    const int off = p - pbase[k], np = npg[k];
+    const int off = p - pbase[k], np = pages_of(k);
     h = off / np;
     g = off % np;
   };
@@ -114,7 +115,7 @@ __global__ void __launch_bounds__(ATT_THREADS) k_attn_decode(ModelDims md, StepD
       int k, h, g;
       locate(p0, k, h, g);
       int slot = s.slots[s.idx[r * maxB + k]];
-      int L = s.len[slot * M + r] + 1;
+      int L = nkeys[k];
       for (int p = p0; p < p1; ++p) {
         const int i = p - p0, st = i % S::NST;
         if (i >= S::NST && (*abort_flag || !mbar_wait(smem_u32(&empty[st]), ((i / S::NST) - 1) & 1, s.err))) {
@@ -135,13 +136,16 @@ __global__ void __launch_bounds__(ATT_THREADS) k_attn_decode(ModelDims md, StepD
           bulk_g2s(smem_u32(dst), pg + ((size_t)(j * 2 + 0) * Hkv + h) * ATT_PS * HD, bytes, bar);
           bulk_g2s(smem_u32(dst + S::SEG_BYTES), pg + ((size_t)(j * 2 + 1) * Hkv + h) * ATT_PS * HD, bytes, bar);
         }
-        if (++g == npg[k]) {
+        if (++g == pages_of(k)) {
           g = 0;
           if (++h == Hkv) {
             h = 0;
-            if (++k < n_r) {
+            do {
+              ++k;
+            } while (k < n_r && nkeys[k] == 0);  // rows with no keys have no pages (no gather)
+            if (k < n_r) {
               slot = s.slots[s.idx[r * maxB + k]];
-              L = s.len[slot * M + r] + 1;
+              L = nkeys[k];
             }
           }
         }
@@ -159,8 +163,7 @@ __global__ void __launch_bounds__(ATT_THREADS) k_attn_decode(ModelDims md, StepD
   float q[G][S::VEC];
   float run_m[G], run_l[G], acc[G][S::VEC];
   auto begin_item = [&]() {
-    const int slot = s.slots[s.idx[r * maxB + k]];
-    L = s.len[slot * M + r] + 1;
+    L = nkeys[k];
     const float* qrow = Q + (size_t)k * md.Hq * HD;
 #pragma unroll
     for (int gg = 0; gg < G; ++gg) {
@@ -236,7 +239,7 @@ __global__ void __launch_bounds__(ATT_THREADS) k_attn_decode(ModelDims md, StepD
     __syncwarp();
     if (lane == 0) mbar_arrive(smem_u32(&empty[st]));
 
-    const bool item_end = (g + 1 == npg[k]);
+    const bool item_end = (g + 1 == pages_of(k));
     if (item_end || p + 1 == p1) {
       // ---- this CTA's part of item (k, h) is done: merge the lane groups, then the warps ----
 #pragma unroll
@@ -261,7 +264,7 @@ __global__ void __launch_bounds__(ATT_THREADS) k_attn_decode(ModelDims md, StepD
         }
       }
       consumer_sync();
-      const int np = npg[k];
+      const int np = pages_of(k);
       const int item = k * Hkv + h;
       const int first = pbase[k] + h * np;
       const int c_first = first / per, c_last = (first + np - 1) / per;
@@ -324,7 +327,9 @@ __global__ void __launch_bounds__(ATT_THREADS) k_attn_decode(ModelDims md, StepD
         g = 0;
         if (++h == Hkv) {
           h = 0;
-          ++k;
+          do {
+            ++k;
+          } while (k < n_r && nkeys[k] == 0);
         }
         begin_item();
       }

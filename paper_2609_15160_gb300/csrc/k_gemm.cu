@@ -37,6 +37,7 @@ __device__ __forceinline__ void gemm_write(const GemmArgs& a, int split, int row
   if (a.epi == EPI_PARTIAL) {
     a.out[((size_t)split * a.max_rows + row) * a.N + col] = v;
   } else if (a.epi == EPI_RESID) {
+    if (a.act && !a.act[row]) return;  // masked row (no-gather ablation): residual unchanged
     const int r = a.idx ? a.idx[row] : row;
     atomicAdd(a.resid + (size_t)r * a.ldr + col, v);
   } else {
@@ -111,7 +112,7 @@ __device__ void cluster_epilogue(const GemmArgs& a, float* red, int4* ci, int m0
 #pragma unroll
         for (int q = 0; q < 4; ++q)
           if (c + q < c1)  // the only writer of this element
-            atomicAdd(a.resid + (size_t)ci[c + q].w * a.ldr + col, sm[q]);
+            if (ci[c + q].w >= 0) atomicAdd(a.resid + (size_t)ci[c + q].w * a.ldr + col, sm[q]);
       }
     return;
   }
@@ -295,7 +296,9 @@ __global__ void __launch_bounds__(128) k_gemm_tc(const __grid_constant__ CUtenso
         if (a.epi == EPI_CL_QKV && !a.row_cslot) {
           colinfo[c] = a.s.rowinfo[a.r * a.md.max_batch + tok0 + c];
         } else if (a.epi == EPI_CL_RESID) {
-          colinfo[c] = make_int4(0, 0, 0, a.idx ? a.idx[tok0 + c] : tok0 + c);
+          // residual row; -1 for a row masked by the no-gather ablation (residual unchanged)
+          const bool masked = a.act && !a.act[tok0 + c];
+          colinfo[c] = make_int4(0, 0, 0, masked ? -1 : (a.idx ? a.idx[tok0 + c] : tok0 + c));
         }
       }
     }

@@ -111,10 +111,9 @@ __global__ void __launch_bounds__(256) k_rope_append(ModelDims md, StepDev s, in
   if (t >= n_pairs + md.Hkv * md.hd) return;
   // page, slot and position of the token's new loop-r entry, from the plan kernel
   const int4 ri = s.rowinfo[r * md.max_batch + k];
-  const int page = ri.x, off = ri.y, pos = ri.z;
-  if (page < 0) return;
+  const int page = ri.x, off = ri.y, pos = ri.z;  // page -1: q only (no append target)
   const int ps = md.page_size, hd = md.hd, half = hd / 2;
-  T* pg = reinterpret_cast<T*>(s.pool) + (size_t)page * md.page_elems;
+  T* pg = reinterpret_cast<T*>(s.pool) + (size_t)(page < 0 ? 0 : page) * md.page_elems;
   const size_t pstride = (size_t)md.max_batch * md.qkv_dim;
   const float* prow = part + (size_t)k * md.qkv_dim;
 
@@ -133,12 +132,12 @@ __global__ void __launch_bounds__(256) k_rope_append(ModelDims md, StepDev s, in
       float* qo = Q + ((size_t)k * md.Hq + h) * hd;
       qo[i] = ra;
       qo[i + half] = rc;
-    } else {
+    } else if (page >= 0) {
       T* kp = pg + ((size_t)(j * 2 + 0) * md.Hkv + (h - md.Hq)) * ps * hd + (size_t)off * hd;
       kp[i] = from_f32<T>(ra);
       kp[i + half] = from_f32<T>(rc);
     }
-  } else {
+  } else if (page >= 0) {
     const int tv = t - n_pairs;
     const int h = tv / hd, e = tv % hd;
     const int col = md.q_dim + md.kv_dim + tv;

@@ -161,6 +161,8 @@ __global__ void __launch_bounds__(256) k_plan(ModelDims md, StepDev s, int B) {
   const int maxB = md.max_batch, M = md.M, ps = md.page_size;
   // attention merge tickets start at zero every step
   for (int i = b; i < maxB * md.Hkv; i += blockDim.x) s.cnt[i] = 0;
+  // without the gather (an ablation), every row of the step is listed at every loop that runs
+  const bool all_rows = md.ablation == TLF_ABLATION_NO_GATHER;
   for (int r = 0; r < M; ++r) {
     const bool active = mb > r;
     // compaction: ballot gives each active lane its rank in the warp, the block scan the warp offsets
@@ -168,37 +170,46 @@ __global__ void __launch_bounds__(256) k_plan(ModelDims md, StepDev s, int B) {
     const int rank = __popc(ball & ((1u << lane) - 1u));
     int n_r;
     const int warp_off = block_exclusive_scan((lane == 0) ? __popc(ball) : 0, &n_r);
-    const int k = __shfl_sync(0xffffffffu, warp_off, 0) + rank;
-    if (active) s.idx[r * maxB + k] = b;
-    // attention plan over the loop-r caches (the token's own new entry included): every
-    // (token, kv head) item spans np pages; items are laid out token-major in one flat page order
-    const int L = active ? s.len[slot * M + r] + 1 : 0;
+    const int n_list = all_rows ? (n_r > 0 ? B : 0) : n_r;
+    const bool listed = all_rows ? (b < B && n_r > 0) : active;
+    const int k = all_rows ? b : __shfl_sync(0xffffffffu, warp_off, 0) + rank;
+    if (listed) {
+      s.idx[r * maxB + k] = b;
+      if (s.act) s.act[r * maxB + k] = active ? 1 : 0;
+    }
+    // attention plan over the loop-r caches: an active token attends to its cache including its own
+    // new entry; a masked row (no gather) to the entries already there. Every (token, kv head) item
+    // spans ceil(keys / page) pages; items are laid out token-major in one flat page order
+    const int L = listed ? s.len[slot * M + r] + (active ? 1 : 0) : 0;
     const int np = (L + ps - 1) / ps;
     int pages;
     const int base = block_exclusive_scan(np * md.Hkv, &pages);
-    if (active) {
+    if (listed) {
       s.item_base[r * (maxB + 1) + k] = base;
-      s.nch[r * maxB + k] = np;
+      s.nch[r * maxB + k] = L;
     }
-    if (active && s.rowinfo) {  // NULL for callers that only attend (no append this step)
-      // where the token's k, v go (Eq. 11): slot L - 1 of the loop-r cache, at its original
-      // position (its loop-1 length, since every token runs loop 1); the position table of the
-      // page is filled here once for all layers
-      const int e = L - 1;
-      int pos = s.len[slot * M];
-      int page = s.page_table[((size_t)slot * M + r) * md.max_pages + e / ps];
-      if (page < 0 || page >= md.n_pages || pos >= md.max_pos) {
-        atomicOr(s.err, DEVERR_INDEX);
-        page = -1;
-        pos = 0;
-      } else {
-        s.pos_table[(size_t)page * ps + e % ps] = pos;
+    if (listed && s.rowinfo) {  // NULL for callers that only attend (no append this step)
+      int page = -1, e = 0, pos = 0;
+      if (active) {
+        // where the token's k, v go (Eq. 11): slot L - 1 of the loop-r cache, at its original
+        // position (its loop-1 length, since every token runs loop 1); the position table of the
+        // page is filled here once for all layers
+        e = L - 1;
+        pos = s.len[slot * M];
+        page = s.page_table[((size_t)slot * M + r) * md.max_pages + e / ps];
+        if (page < 0 || page >= md.n_pages || pos >= md.max_pos) {
+          atomicOr(s.err, DEVERR_INDEX);
+          page = -1;
+          pos = 0;
+        } else {
+          s.pos_table[(size_t)page * ps + e % ps] = pos;
+        }
       }
-      s.rowinfo[r * maxB + k] = make_int4(page, e % ps, pos, 0);
+      s.rowinfo[r * maxB + k] = make_int4(page, e % ps, pos, b);
     }
     if (b == 0) {
-      s.n[r] = n_r;
-      s.item_base[r * (maxB + 1) + n_r] = pages;
+      s.n[r] = n_list;
+      s.item_base[r * (maxB + 1) + n_list] = pages;
       s.chunk[r] = ps;
     }
   }

@@ -65,6 +65,7 @@ struct tlf_ctx {
   double* d_inv_freq = nullptr;
   float2* d_rope = nullptr;     // [max_pos][hd/2] (cos, sin)
   int4* d_rowinfo = nullptr;    // [M][max_batch]
+  int* d_act = nullptr;         // [M][max_batch]
   std::vector<DeviceMat> wqkv, wo, wgu, wd;
   DeviceMat emb_mat;
 
@@ -222,6 +223,8 @@ extern "C" int tlf_validate_config(const tlf_config* c, char* msg, size_t msg_le
   if (c->kv_pool_pages < 0) return bad("kv_pool_pages must be >= 0");
   if (c->prefill_chunk < 0 || (c->prefill_chunk > 0 && c->prefill_chunk < 64))
     return bad("prefill_chunk must be 0 (default) or >= 64");
+  if (c->ablation != TLF_ABLATION_NONE && c->ablation != TLF_ABLATION_NO_GATHER) return bad("unknown ablation");
+  if (c->reserved != 0) return bad("reserved must be 0");
   if (msg && msg_len) snprintf(msg, msg_len, "ok");
   return TLF_OK;
 }
@@ -328,6 +331,7 @@ static int create_impl(tlf_ctx* ctx, const tlf_weights* w) {
   md.eps = c.norm_eps; md.rope_base = c.rope_base; md.threshold = c.threshold; md.exit_rule = c.exit_rule;
   md.dtype = c.dtype;
   md.max_pos = c.max_seq_len;
+  md.ablation = c.ablation;
   ctx->eb = c.dtype == TLF_DTYPE_BF16 ? 2 : 4;
   md.page_elems = (long long)md.J * 2 * md.Hkv * md.page_size * md.hd;
   ctx->n_pages = c.kv_pool_pages > 0 ? c.kv_pool_pages : (int64_t)c.max_seqs * c.max_loops * md.max_pages;
@@ -484,6 +488,7 @@ static int create_impl(tlf_ctx* ctx, const tlf_weights* w) {
     return rc;
   if ((rc = dev_alloc(ctx, &ctx->d_attn_cnt, (size_t)B * md.Hkv * 4, "attention tickets"))) return rc;
   if ((rc = dev_alloc(ctx, &ctx->d_rowinfo, (size_t)M * B * sizeof(int4), "row info"))) return rc;
+  if ((rc = dev_alloc(ctx, &ctx->d_act, (size_t)M * B * 4, "row masks"))) return rc;
   CK(ctx, cudaMemset(ctx->d_attn_cnt, 0, (size_t)B * md.Hkv * 4));
   if ((rc = dev_alloc(ctx, &ctx->d_logits, (size_t)B * V * 4, "logits"))) return rc;
   if ((rc = dev_alloc(ctx, &ctx->d_err, 16, "error word"))) return rc;
@@ -508,7 +513,7 @@ extern "C" void tlf_destroy(tlf_ctx* ctx) {
     cudaDeviceSynchronize();
     auto f = [](void* p) { if (p) cudaFree(p); };
     f(ctx->d_emb); f(ctx->d_router_w); f(ctx->d_router_b); f(ctx->d_attn_norm); f(ctx->d_mlp_norm);
-    f(ctx->d_final_norm); f(ctx->d_inv_freq); f(ctx->d_rope); f(ctx->d_rowinfo);
+    f(ctx->d_final_norm); f(ctx->d_inv_freq); f(ctx->d_rope); f(ctx->d_rowinfo); f(ctx->d_act);
     for (auto* v : {&ctx->wqkv, &ctx->wo, &ctx->wgu, &ctx->wd})
       for (auto& m : *v) f(m.ptr);
     f(ctx->d_pool); f(ctx->d_pos_table); f(ctx->d_page_table); f(ctx->d_len); f(ctx->d_upload);
@@ -669,6 +674,7 @@ static int enqueue_step(tlf_ctx* ctx, int B, bool need_logits, bool prof, cudaSt
   s.err = ctx->d_err;
   s.cnt = ctx->d_attn_cnt;
   s.rowinfo = ctx->d_rowinfo;
+  s.act = ctx->d_act;
   const PageUpdate* d_upd = reinterpret_cast<const PageUpdate*>(ctx->d_upload + 1 + 3 * B);
 
   ctx->last_launches = 0;
@@ -689,6 +695,8 @@ static int enqueue_step(tlf_ctx* ctx, int B, bool need_logits, bool prof, cudaSt
   for (int r = 0; r < M; ++r) {
     const int* n_dev = ctx->d_n + r;
     const int* idx_r = ctx->d_idx + (size_t)r * maxB;
+    // rows that do not run loop r but are computed anyway (no-gather ablation) keep their residual
+    const int* act_r = md.ablation == TLF_ABLATION_NO_GATHER ? ctx->d_act + (size_t)r * maxB : nullptr;
     for (int j = 0; j < J; ++j) {
       launch_norm_rows(md.dtype, ctx->d_H, md.d, idx_r, n_dev, 0, maxB, ctx->d_attn_norm + (size_t)j * md.d, md.d,
                        md.eps, ctx->d_X, md.d, st);
@@ -726,6 +734,7 @@ static int enqueue_step(tlf_ctx* ctx, int B, bool need_logits, bool prof, cudaSt
       a.resid = ctx->d_H;
       a.ldr = md.d;
       a.idx = idx_r;
+      a.act = act_r;
       a.splits = ctx->s_o;
       gemm(ctx, ctx->wo[j], &ctx->map_O, ctx->d_O, md.q_dim, a, st);
       mark(6);
@@ -758,6 +767,7 @@ static int enqueue_step(tlf_ctx* ctx, int B, bool need_logits, bool prof, cudaSt
       a.resid = ctx->d_H;
       a.ldr = md.d;
       a.idx = idx_r;
+      a.act = act_r;
       a.splits = ctx->s_d;
       gemm(ctx, ctx->wd[j], &ctx->map_U, ctx->d_U, md.ff, a, st);
       mark(10);
@@ -850,11 +860,15 @@ static int run_step(tlf_ctx* ctx, int B, const int* slots, const int* tokens, co
       ctx->class_ms[ctx->ev_class[i]] += ms;
     }
     ctx->last_attn_ms = ctx->class_ms[5];
-    // KV bytes visited: for every row b and loop r < m_b, (len + 1) entries x J layers x K,V
+    // KV bytes visited: for every row b and loop r < m_b, (len + 1) entries x J layers x K,V;
+    // without the gather, every loop that runs also reads the caches of the exited rows
     double bytes = 0.0;
+    int loops_run = 0;
+    for (int b = 0; b < B; ++b) loops_run = std::max(loops_run, ctx->h_m[b]);
     for (int b = 0; b < B; ++b)
-      for (int r = 0; r < ctx->h_m[b]; ++r)
-        bytes += (double)(ctx->h_len[(size_t)slots[b] * M + r] + 1) * J * 2.0 * md.Hkv * md.hd * ctx->eb;
+      for (int r = 0; r < (md.ablation == TLF_ABLATION_NO_GATHER ? loops_run : ctx->h_m[b]); ++r)
+        bytes += (double)(ctx->h_len[(size_t)slots[b] * M + r] + (r < ctx->h_m[b] ? 1 : 0)) * J * 2.0 * md.Hkv *
+                 md.hd * ctx->eb;
     ctx->last_attn_bytes = bytes;
   }
   ctx->last_batch = B;

@@ -308,7 +308,9 @@ struct StepDev {
   int* idx;            // [M][maxB] rows of A_r in increasing order
   int* n;              // [M] |A_r|
   int* item_base;      // [M][maxB+1]
-  int* nch;            // [M][maxB] chunks per token
+  int* nch;            // [M][maxB] keys each kv head of the token attends to (0: no work)
+  int* act;            // [M][maxB] 1 if compact row k runs loop r (always, except rows masked
+                       // by TLF_ABLATION_NO_GATHER)
   int* chunk;          // [M] keys per page
   int* cnt;            // [maxB * Hkv] attention merge tickets (zeroed by the plan kernel)
   int4* rowinfo;       // [M][maxB] per compact row k of A_r: {page, slot in page, position, 0} of the
@@ -332,6 +334,7 @@ struct ModelDims {
   int exit_rule;
   int dtype;             // 0 f32, 1 bf16
   int max_pos;           // positions 0..max_pos-1 have a row in the rotary table
+  int ablation;          // tlf_ablation
 };
 
 struct GemmArgs {
@@ -339,6 +342,7 @@ struct GemmArgs {
   int K;             // reduction length
   int splits;        // split-K factor (gridDim.y; the cluster size for EPI_CL_*)
   int stages;        // depth of the tcgen05 kernel's operand ring (set by the launcher)
+  const int* act;    // RESID epilogues: rows with act[row] == 0 keep their residual (NULL: none)
   const int* n_dev;  // token rows n (device scalar), or NULL to use n_host
   int n_host;
   int epi;           // GemmEpilogue

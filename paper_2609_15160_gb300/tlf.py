@@ -25,6 +25,7 @@ KERNEL_CLASSES = ("router", "plan", "attn_norm", "qkv_gemm", "rope_append", "att
 DTYPE = {"f32": 0, "bf16": 1}
 EXIT = {"argmax": 0, "survival": 1}
 GEMM = {"auto": 0, "simt": 1}
+ABLATION = {"none": 0, "no_gather": 1}
 
 
 class TlfConfig(C.Structure):
@@ -33,7 +34,7 @@ class TlfConfig(C.Structure):
         ("rope_base", C.c_float), ("norm_eps", C.c_float), ("dtype", C.c_int32), ("exit_rule", C.c_int32),
         ("threshold", C.c_float), ("max_seqs", C.c_int32), ("max_batch", C.c_int32), ("max_seq_len", C.c_int32),
         ("page_size", C.c_int32), ("gemm_impl", C.c_int32), ("host_only", C.c_int32), ("prefill_chunk", C.c_int32),
-        ("kv_pool_pages", C.c_int64)]
+        ("kv_pool_pages", C.c_int64), ("ablation", C.c_int32), ("reserved", C.c_int32)]
 
 
 class TlfWeights(C.Structure):
@@ -139,13 +140,13 @@ def _stream(stream) -> Optional[int]:
 
 def make_config(m, max_seqs: int, max_batch: int, max_seq_len: int, page_size: int = 64,
                 kv_pool_pages: int = 0, gemm_impl: str = "auto", host_only: bool = False,
-                prefill_chunk: int = 0) -> TlfConfig:
+                prefill_chunk: int = 0, ablation: str = "none") -> TlfConfig:
     return TlfConfig(vocab=m.vocab, d_model=m.d_model, n_heads=m.n_heads, n_kv_heads=m.n_kv_heads,
                      head_dim=m.head_dim, n_layers=m.n_layers, ffn_hidden=m.ffn_hidden, max_loops=m.max_loops,
                      rope_base=m.rope_base, norm_eps=m.norm_eps, dtype=DTYPE[m.dtype], exit_rule=EXIT[m.exit_rule],
                      threshold=m.threshold, max_seqs=max_seqs, max_batch=max_batch, max_seq_len=max_seq_len,
                      page_size=page_size, gemm_impl=GEMM[gemm_impl], host_only=int(host_only), prefill_chunk=prefill_chunk,
-                     kv_pool_pages=kv_pool_pages)
+                     kv_pool_pages=kv_pool_pages, ablation=ABLATION[ablation])
 
 
 def tlf_validate_config(cfg: TlfConfig):
@@ -244,10 +245,11 @@ class Context:
 
     def __init__(self, model, weights: Optional[Dict[str, np.ndarray]], max_seqs: int, max_batch: int,
                  max_seq_len: int, kv_pool_pages: int = 0, gemm_impl: str = "auto", host_only: bool = False,
-                 prefill_chunk: int = 0):
+                 prefill_chunk: int = 0, ablation: str = "none"):
         self.model = model
         self.cfg = make_config(model, max_seqs, max_batch, max_seq_len, kv_pool_pages=kv_pool_pages,
-                               gemm_impl=gemm_impl, host_only=host_only, prefill_chunk=prefill_chunk)
+                               gemm_impl=gemm_impl, host_only=host_only, prefill_chunk=prefill_chunk,
+                               ablation=ablation)
         self.handle, _ = tlf_create(self.cfg, weights, model.dtype)
         self.max_batch = max_batch
 

@@ -45,10 +45,17 @@ class DepthOracle:
         return m
 
 
-def check_active_sets(ctx, loops, M):
+def check_active_sets(ctx, loops, M, ablation="none"):
+    """The rows each loop ran on: A_r = {b : m_b >= r} in increasing b (Eq. 4-6).
+
+    Without the gather (the no-gather ablation) every loop that has an active
+    token lists all rows of the step instead.
+    """
     counts, sets = ctx.last_active_sets(len(loops))
     for r in range(M):
         want = np.nonzero(loops >= r + 1)[0]
+        if ablation == "no_gather" and want.size:
+            want = np.arange(len(loops))
         assert counts[r] == want.size, (r, counts[r], want.size)
         np.testing.assert_array_equal(sets[r], want)
 

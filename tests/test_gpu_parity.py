@@ -24,7 +24,7 @@ def tlf():
     return T
 
 
-def _greedy_run(T, wl, steps=None, gemm_impl="auto", check_caches=True):
+def _greedy_run(T, wl, steps=None, gemm_impl="auto", check_caches=True, ablation="none"):
     """Prefill + greedy decode, teacher-forced from the oracle's argmax."""
     m = wl.model
     w = synth.make_weights(m)
@@ -37,7 +37,7 @@ def _greedy_run(T, wl, steps=None, gemm_impl="auto", check_caches=True):
     ids = list(range(100, 100 + B))
     tol = tol_for(m)
     worst = 0.0
-    with T.Context(m, w, max_seqs=B, max_batch=B, max_seq_len=L, gemm_impl=gemm_impl) as ctx:
+    with T.Context(m, w, max_seqs=B, max_batch=B, max_seq_len=L, gemm_impl=gemm_impl, ablation=ablation) as ctx:
         pf_forced = [depth.forced_for(p) for p in prompts]
         glog, gloops = ctx.prefill(ids, prompts, forced=pf_forced)
         seqs = [O.OracleSequence(om) for _ in range(B)]
@@ -54,7 +54,7 @@ def _greedy_run(T, wl, steps=None, gemm_impl="auto", check_caches=True):
             glog, gl, gmar = ctx.decode_step(ids, nxt, forced=f)
             olog, oloops, omar = O.decode_step(om, seqs, nxt, forced=f)
             np.testing.assert_array_equal(gl, oloops)
-            check_active_sets(ctx, gl, m.max_loops)
+            check_active_sets(ctx, gl, m.max_loops, ablation)
             e = rel_err(glog, olog)
             worst = max(worst, e)
             assert e < tol, f"step {step}: logits rel err {e}"
@@ -86,7 +86,7 @@ def test_c2_simt_gemm_path_matches_oracle(tlf):
     print(f"c2 simt worst {worst:.2e}")
 
 
-def _snapshot_run(T, wl, lengths, steps, sampled, seed=7, distinct=2):
+def _snapshot_run(T, wl, lengths, steps, sampled, seed=7, distinct=2, ablation="none"):
     """Sequences restored from synthetic cache snapshots, then decode steps of random tokens.
 
     Loop counts and active sets are checked for every token (against the
@@ -109,7 +109,7 @@ def _snapshot_run(T, wl, lengths, steps, sampled, seed=7, distinct=2):
     tol = tol_for(m)
     worst = 0.0
     with T.Context(m, w, max_seqs=B, max_batch=B, max_seq_len=int(max(lengths)) + steps + 1,
-                   kv_pool_pages=pages) as ctx:
+                   kv_pool_pages=pages, ablation=ablation) as ctx:
         for b in range(B):
             ctx.load_cache(ids[b], snaps[(int(lengths[b]), b % distinct)])
         oseqs = {b: O.load_snapshot(om, snaps[(int(lengths[b]), b % distinct)], cache_dtype=np.float32)
@@ -119,7 +119,7 @@ def _snapshot_run(T, wl, lengths, steps, sampled, seed=7, distinct=2):
             f = depth.forced_for(tokens[step])
             glog, gl, _ = ctx.decode_step(ids, tokens[step], forced=f)
             np.testing.assert_array_equal(gl, depth.expected(tokens[step], f))
-            check_active_sets(ctx, gl, m.max_loops)
+            check_active_sets(ctx, gl, m.max_loops, ablation)
             all_loops.append(gl.copy())
             for b in sampled:
                 olog, oml, _ = O.decode_token(om, oseqs[b], int(tokens[step][b]), forced=int(f[b]))
@@ -173,7 +173,7 @@ def _small(dtype="bf16", **kw):
     return synth.ModelConfig(**base)
 
 
-def _prefill_decode_compare(T, m, prompt_lens, steps, forced_mode=None, seed=0, gemm_impl="auto"):
+def _prefill_decode_compare(T, m, prompt_lens, steps, forced_mode=None, seed=0, gemm_impl="auto", ablation="none"):
     w = synth.make_weights(m)
     om = O.OracleModel.from_config(m, w)
     depth = DepthOracle(om)
@@ -191,7 +191,7 @@ def _prefill_decode_compare(T, m, prompt_lens, steps, forced_mode=None, seed=0, 
         return np.full(len(toks), forced_mode, dtype=np.int32)
 
     with T.Context(m, w, max_seqs=B + 1, max_batch=B, max_seq_len=max(prompt_lens) + steps + 2,
-                   gemm_impl=gemm_impl) as ctx:
+                   gemm_impl=gemm_impl, ablation=ablation) as ctx:
         pf = [forced_of(p) for p in prompts]
         glog, gl = ctx.prefill(ids, prompts, forced=pf)
         seqs = [O.OracleSequence(om) for _ in range(B)]
@@ -205,7 +205,7 @@ def _prefill_decode_compare(T, m, prompt_lens, steps, forced_mode=None, seed=0, 
             glog, gm, _ = ctx.decode_step(ids, toks, forced=f)
             olog, om2, _ = O.decode_step(om, seqs, toks, forced=f)
             np.testing.assert_array_equal(gm, om2)
-            check_active_sets(ctx, gm, m.max_loops)
+            check_active_sets(ctx, gm, m.max_loops, ablation)
             assert rel_err(glog, olog) < tol
         for b in range(B):
             check_cache(ctx, ids[b], seqs[b], m)
@@ -340,3 +340,28 @@ def test_decode_step_is_deterministic(tlf):
             outs.append(res)
     for a, b in zip(*outs):
         np.testing.assert_array_equal(a, b)
+
+
+# ----------------------------------------------------------------------------
+# ablations: the same logits and loop counts as the method, different work
+# ----------------------------------------------------------------------------
+
+def test_no_gather_ablation_c2_greedy(tlf):
+    """Without the gather (every loop computes all rows, exited rows masked) the results are the method's."""
+    worst, forced = _greedy_run(tlf, synth.get_config("c2"), steps=24, ablation="no_gather")
+    print(f"c2 no-gather worst {worst:.2e} forced {forced}")
+
+
+@pytest.mark.parametrize("gemm_impl", ["auto", "simt"])
+@pytest.mark.parametrize("lens", [[1, 64, 65], [130, 2, 70, 64]])
+def test_no_gather_ablation_edges(tlf, lens, gemm_impl):
+    """Rows that exit with empty deeper caches (no keys at all) and page boundaries."""
+    _prefill_decode_compare(tlf, _small(), lens, steps=4, gemm_impl=gemm_impl, ablation="no_gather")
+
+
+def test_no_gather_ablation_c5_ragged(tlf):
+    wl = synth.get_config("c5")
+    lengths = np.array([len(p) for p in synth.make_prompts(wl)])
+    worst, forced = _snapshot_run(tlf, wl, lengths, steps=2, sampled=[int(np.argmax(lengths)), int(np.argmin(lengths))],
+                                  distinct=1, ablation="no_gather")
+    print(f"c5 no-gather worst {worst:.2e} forced {forced}")
