@@ -202,12 +202,14 @@ def setup_workload(T, wl, rank: int, gemm_impl="auto", prefill="auto", extra_tok
     prompts = synth.make_prompts(wl)
     lengths = [len(p) for p in prompts]
     steps_cap = max(wl.decode_steps, extra_tokens) + 64
-    use_snapshot = prefill == "snapshot"  # default: real (batched) prefill through the library
+    # default: real (batched) prefill through the library. Full-length caches (dense-cache ablation)
+    # prefill position by position, far too slow for long prompts: they restore snapshots instead
+    use_snapshot = prefill == "snapshot" or (prefill == "auto" and ablation == "dense_cache")
     ids = [rank * 100000 + b for b in range(B)]
     if use_snapshot:
         # uniform lengths: two distinct host snapshots (values uploaded); ragged lengths: one
         # snapshot per sequence with only positions, values filled on the device
-        host_values = wl.prompt_len[0] == wl.prompt_len[1]
+        host_values = wl.prompt_len[0] == wl.prompt_len[1] and ablation != "dense_cache"
         distinct = {}
         snaps = []
         for b, L in enumerate(lengths):
@@ -219,6 +221,8 @@ def setup_workload(T, wl, rank: int, gemm_impl="auto", prefill="auto", extra_tok
             snaps.append(distinct[key])
         pages = sum(sum((len(p) + 63) // 64 for p in s["positions"]) for s in snaps) + B * m.max_loops * (
             steps_cap // 64 + 2)
+        if ablation == "dense_cache":  # every loop cache holds a slot per position
+            pages = B * m.max_loops * ((max(lengths) + steps_cap) // 64 + 2)
     else:
         snaps = None
         pages = B * m.max_loops * ((max(lengths) + steps_cap) // 64 + 2)
@@ -500,8 +504,10 @@ def main():
     ap.add_argument("--prefill", default="auto", choices=["auto", "snapshot", "real"])
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--decode-batch", type=int, default=0, help="override the workload's batch (C5 sweep)")
-    ap.add_argument("--ablation", default="none", choices=["none", "no_gather"],
-                    help="decode without the gather of Eq. 6 (all rows every loop, exited rows masked)")
+    ap.add_argument("--ablation", default="none", choices=["none", "no_gather", "dense_cache"],
+                    help="no_gather: all rows every loop, exited rows masked (no gather of Eq. 6); "
+                         "dense_cache: full-length loop caches read under the mask of Eq. 10 "
+                         "(no recursion-wise cache)")
     args = ap.parse_args()
     if args.warmup < 3:
         args.warmup = 3

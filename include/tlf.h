@@ -80,8 +80,16 @@ enum tlf_gemm_impl { TLF_GEMM_AUTO = 0, TLF_GEMM_SIMT = 1 };
  *              all B rows of the step; rows with m <= r are masked: their
  *              residual stream is not updated and they append nothing, but
  *              their projections and attention over their loop-r caches run
- *              (the cost of computing without the gather of Eq. 6). */
-enum tlf_ablation { TLF_ABLATION_NONE = 0, TLF_ABLATION_NO_GATHER = 1 };
+ *              (the cost of computing without the gather of Eq. 6).
+ *   DENSE_CACHE without recursion-wise caches: every loop's cache keeps a slot
+ *              for every position (all M caches have the sequence's length);
+ *              a token that exits before loop r leaves a masked slot there
+ *              (position -1), and attention at loop r reads every slot and
+ *              skips the masked ones (the mask mu^(r) of Eq. 10 applied to a
+ *              full-length cache). bf16 models only; prefill runs position by
+ *              position; tlf_cache_len counts slots and tlf_read_cache returns
+ *              masked slots with position -1. */
+enum tlf_ablation { TLF_ABLATION_NONE = 0, TLF_ABLATION_NO_GATHER = 1, TLF_ABLATION_DENSE_CACHE = 2 };
 
 typedef struct tlf_config {
   int32_t vocab;        /* V; the LM head is tied to the embedding */

@@ -6,6 +6,11 @@
 // storage and the kernel reads no masked slots. The token's own entry was
 // appended before this kernel runs, so the key count is len + 1.
 //
+// Without recursion-wise caches (the dense-cache ablation, MASKED) every loop
+// cache holds a slot per position and slots of tokens that exited earlier are
+// masked (position -1): the kernel then also copies each page's positions and
+// skips masked keys, reading the masked slots' K/V as the ablation requires.
+//
 // Work split (stream-K over pages): an item is one (token, kv head); its keys
 // live in ceil((len+1)/64) pages. The plan kernel lays all items' pages out in
 // one flat order; CTA c of the persistent grid takes the contiguous page range
@@ -25,6 +30,8 @@
 // contributing CTA stores a partial (max, sum, output) and takes a ticket with
 // an atomic counter, and the CTA that takes the last ticket merges the
 // partials and writes the output (no CTA ever waits for another).
+#include <type_traits>
+
 #include "tlf_internal.cuh"
 
 namespace tlf {
@@ -47,17 +54,19 @@ struct AttnShape {
   static_assert(STEPS >= 1, "page too small for the warp split");
 };
 
-template <typename T, int HD, int G>
+// MASKED (the dense-cache ablation): each stage also holds the page's 64 positions, -1 = masked slot.
+template <typename T, int HD, int G, bool MASKED>
 constexpr int attn_smem_bytes() {
   using S = AttnShape<T, HD>;
-  return 128 + S::NST * S::STAGE_BYTES + ATT_WARPS * G * (HD + 2) * 4 + 2 * S::NST * 8 + 16;
+  return 128 + S::NST * S::STAGE_BYTES + ATT_WARPS * G * (HD + 2) * 4 + (MASKED ? S::NST * ATT_PS * 4 : 0) +
+         2 * S::NST * 8 + 16;
 }
 
 __device__ __forceinline__ void consumer_sync() {
   asm volatile("bar.sync 1, %0;" ::"n"(32 * ATT_WARPS) : "memory");
 }
 
-template <typename T, int HD, int G>
+template <typename T, int HD, int G, bool MASKED>
 __global__ void __launch_bounds__(ATT_THREADS) k_attn_decode(ModelDims md, StepDev s, int r, int j,
                                                              const float* __restrict__ Q, float* __restrict__ part,
                                                              T* __restrict__ O, int* __restrict__ cnt) {
@@ -67,7 +76,8 @@ __global__ void __launch_bounds__(ATT_THREADS) k_attn_decode(ModelDims md, StepD
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 127) & ~uintptr_t(127));
   uint8_t* ring = smem;                                                   // [NST][K seg | V seg]
   float* red = reinterpret_cast<float*>(ring + S::NST * S::STAGE_BYTES);  // [warps][G][HD + 2]
-  uint64_t* full = reinterpret_cast<uint64_t*>(red + ATT_WARPS * PSZ);
+  int* mring = reinterpret_cast<int*>(red + ATT_WARPS * PSZ);              // [NST][64] positions (MASKED)
+  uint64_t* full = reinterpret_cast<uint64_t*>(mring + (MASKED ? S::NST * ATT_PS : 0));
   uint64_t* empty = full + S::NST;
   int* flag = reinterpret_cast<int*>(empty + S::NST);
   volatile int* abort_flag = flag + 1;  // set when a bounded wait runs out: later waits are skipped
@@ -132,7 +142,8 @@ __global__ void __launch_bounds__(ATT_THREADS) k_attn_decode(ModelDims md, StepD
           const T* pg = reinterpret_cast<const T*>(s.pool) + (size_t)page * md.page_elems;
           const uint32_t bytes = (uint32_t)(valid * HD * sizeof(T));
           uint8_t* dst = ring + st * S::STAGE_BYTES;
-          mbar_arrive_expect_tx(bar, 2 * bytes);
+          mbar_arrive_expect_tx(bar, 2 * bytes + (MASKED ? ATT_PS * 4 : 0));
+          if (MASKED) bulk_g2s(smem_u32(mring + st * ATT_PS), s.pos_table + (size_t)page * ATT_PS, ATT_PS * 4, bar);
           bulk_g2s(smem_u32(dst), pg + ((size_t)(j * 2 + 0) * Hkv + h) * ATT_PS * HD, bytes, bar);
           bulk_g2s(smem_u32(dst + S::SEG_BYTES), pg + ((size_t)(j * 2 + 1) * Hkv + h) * ATT_PS * HD, bytes, bar);
         }
@@ -184,13 +195,17 @@ __global__ void __launch_bounds__(ATT_THREADS) k_attn_decode(ModelDims md, StepD
     const int valid = min(ATT_PS, L - g * ATT_PS);
     const T* sk = reinterpret_cast<const T*>(ring + st * S::STAGE_BYTES);
     const T* sv = reinterpret_cast<const T*>(ring + st * S::STAGE_BYTES + S::SEG_BYTES);
+    const int* smask = mring + st * ATT_PS;
+    // key slot usable: inside the cache and, for a full-length cache, not masked (mu^(r) of Eq. 10)
+    auto usable = [&](int key) { return key < valid && (!MASKED || smask[key] >= 0); };
 
     float sc[S::STEPS][G];
 #pragma unroll
     for (int t = 0; t < S::STEPS; ++t) {
       const int key = warp * S::KEYS_PER_WARP + t * S::KPW + grp;
       float kv[S::VEC];
-      if (key < valid) {
+      const bool use = usable(key);
+      if (use) {
         Vec16<T>::load(sk + key * HD + part_lane * S::VEC, kv);
       } else {
 #pragma unroll
@@ -203,7 +218,7 @@ __global__ void __launch_bounds__(ATT_THREADS) k_attn_decode(ModelDims md, StepD
         for (int e = 0; e < S::VEC; ++e) d = fmaf(q[gg][e], kv[e], d);
 #pragma unroll
         for (int o = S::LPK / 2; o > 0; o >>= 1) d += __shfl_xor_sync(0xffffffffu, d, o);
-        sc[t][gg] = (key < valid) ? d : -INFINITY;
+        sc[t][gg] = use ? d : -INFINITY;
       }
     }
 #pragma unroll
@@ -224,7 +239,7 @@ __global__ void __launch_bounds__(ATT_THREADS) k_attn_decode(ModelDims md, StepD
 #pragma unroll
     for (int t = 0; t < S::STEPS; ++t) {
       const int key = warp * S::KEYS_PER_WARP + t * S::KPW + grp;
-      if (key < valid) {
+      if (usable(key)) {
         float vv[S::VEC];
         Vec16<T>::load(sv + key * HD + part_lane * S::VEC, vv);
 #pragma unroll
@@ -339,16 +354,28 @@ __global__ void __launch_bounds__(ATT_THREADS) k_attn_decode(ModelDims md, StepD
   }
 }
 
+template <typename T, int HD, int G, bool MASKED>
+static void attn_launch_v(const ModelDims& md, const StepDev& s, int r, int j, const float* Q, float* part, void* O,
+                          int* cnt, int grid, cudaStream_t st) {
+  static bool attr = false;
+  constexpr int smem = attn_smem_bytes<T, HD, G, MASKED>();
+  if (!attr) {
+    cudaFuncSetAttribute(k_attn_decode<T, HD, G, MASKED>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+    attr = true;
+  }
+  launch_k(k_attn_decode<T, HD, G, MASKED>, grid, ATT_THREADS, smem, st, md, s, r, j, Q, part, (T*)O, cnt);
+}
+
 template <typename T, int HD, int G>
 static void attn_launch(const ModelDims& md, const StepDev& s, int r, int j, const float* Q, float* part, void* O,
                         int* cnt, int grid, cudaStream_t st) {
-  static bool attr = false;
-  constexpr int smem = attn_smem_bytes<T, HD, G>();
-  if (!attr) {
-    cudaFuncSetAttribute(k_attn_decode<T, HD, G>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
-    attr = true;
+  if constexpr (std::is_same<T, bf16>::value) {
+    if (md.ablation == TLF_ABLATION_DENSE_CACHE) {
+      attn_launch_v<T, HD, G, true>(md, s, r, j, Q, part, O, cnt, grid, st);
+      return;
+    }
   }
-  launch_k(k_attn_decode<T, HD, G>, grid, ATT_THREADS, smem, st, md, s, r, j, Q, part, (T*)O, cnt);
+  attn_launch_v<T, HD, G, false>(md, s, r, j, Q, part, O, cnt, grid, st);
 }
 
 #define TLF_ATTN_DISPATCH(FN, ...)                                                              \

@@ -199,8 +199,10 @@ __global__ void __launch_bounds__(256) k_final(ModelDims md, StepDev s, const fl
   const float inv = rsqrtf(ss / (float)md.d + md.eps);
   for (int i = threadIdx.x; i < md.d; i += blockDim.x) Xf[(size_t)b * md.d + i] = from_f32<T>(h[i] * inv * gain[i]);
   if (threadIdx.x < md.M) {
+    // every loop cache the token wrote to grows by one (all of them without recursion-wise caches,
+    // where the loops it skipped hold a masked slot)
     const int r = threadIdx.x;
-    if (r < s.m[b]) s.len[s.slots[b] * md.M + r] += 1;
+    if (r < s.m[b] || md.ablation == TLF_ABLATION_DENSE_CACHE) s.len[s.slots[b] * md.M + r] += 1;
   }
 }
 

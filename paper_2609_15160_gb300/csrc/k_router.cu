@@ -163,6 +163,7 @@ __global__ void __launch_bounds__(256) k_plan(ModelDims md, StepDev s, int B) {
   for (int i = b; i < maxB * md.Hkv; i += blockDim.x) s.cnt[i] = 0;
   // without the gather (an ablation), every row of the step is listed at every loop that runs
   const bool all_rows = md.ablation == TLF_ABLATION_NO_GATHER;
+  const bool dense = md.ablation == TLF_ABLATION_DENSE_CACHE;
   for (int r = 0; r < M; ++r) {
     const bool active = mb > r;
     // compaction: ballot gives each active lane its rank in the warp, the block scan the warp offsets
@@ -206,6 +207,14 @@ __global__ void __launch_bounds__(256) k_plan(ModelDims md, StepDev s, int B) {
         }
       }
       s.rowinfo[r * maxB + k] = make_int4(page, e % ps, pos, b);
+    }
+    if (dense && b < B && !active && s.rowinfo) {
+      // no recursion-wise cache (an ablation): the exited token still takes its slot in the loop-r
+      // cache, masked with position -1, so every loop's cache keeps one slot per position
+      const int e = s.len[slot * M + r];
+      const int page = s.page_table[((size_t)slot * M + r) * md.max_pages + e / ps];
+      if (page < 0 || page >= md.n_pages) atomicOr(s.err, DEVERR_INDEX);
+      else s.pos_table[(size_t)page * ps + e % ps] = -1;
     }
     if (b == 0) {
       s.n[r] = n_list;

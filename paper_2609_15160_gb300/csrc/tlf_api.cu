@@ -223,7 +223,11 @@ extern "C" int tlf_validate_config(const tlf_config* c, char* msg, size_t msg_le
   if (c->kv_pool_pages < 0) return bad("kv_pool_pages must be >= 0");
   if (c->prefill_chunk < 0 || (c->prefill_chunk > 0 && c->prefill_chunk < 64))
     return bad("prefill_chunk must be 0 (default) or >= 64");
-  if (c->ablation != TLF_ABLATION_NONE && c->ablation != TLF_ABLATION_NO_GATHER) return bad("unknown ablation");
+  if (c->ablation != TLF_ABLATION_NONE && c->ablation != TLF_ABLATION_NO_GATHER &&
+      c->ablation != TLF_ABLATION_DENSE_CACHE)
+    return bad("unknown ablation");
+  if (c->ablation == TLF_ABLATION_DENSE_CACHE && c->dtype != TLF_DTYPE_BF16)
+    return bad("the dense-cache ablation needs a bf16 model");
   if (c->reserved != 0) return bad("reserved must be 0");
   if (msg && msg_len) snprintf(msg, msg_len, "ok");
   return TLF_OK;
@@ -866,9 +870,13 @@ static int run_step(tlf_ctx* ctx, int B, const int* slots, const int* tokens, co
     int loops_run = 0;
     for (int b = 0; b < B; ++b) loops_run = std::max(loops_run, ctx->h_m[b]);
     for (int b = 0; b < B; ++b)
-      for (int r = 0; r < (md.ablation == TLF_ABLATION_NO_GATHER ? loops_run : ctx->h_m[b]); ++r)
-        bytes += (double)(ctx->h_len[(size_t)slots[b] * M + r] + (r < ctx->h_m[b] ? 1 : 0)) * J * 2.0 * md.Hkv *
-                 md.hd * ctx->eb;
+      for (int r = 0; r < (md.ablation == TLF_ABLATION_NO_GATHER ? loops_run : ctx->h_m[b]); ++r) {
+        const double keys = ctx->h_len[(size_t)slots[b] * M + r] + (r < ctx->h_m[b] ? 1 : 0);
+        bytes += keys * J * 2.0 * md.Hkv * md.hd * ctx->eb;
+        // a full-length cache (dense-cache ablation) also reads each page's 64 positions per kv head
+        if (md.ablation == TLF_ABLATION_DENSE_CACHE)
+          bytes += std::ceil(keys / md.page_size) * J * md.Hkv * md.page_size * 4.0;
+      }
     ctx->last_attn_bytes = bytes;
   }
   ctx->last_batch = B;
@@ -877,8 +885,9 @@ static int run_step(tlf_ctx* ctx, int B, const int* slots, const int* tokens, co
 
 static void advance_lengths(tlf_ctx* ctx, int B, const int* slots) {
   const int M = ctx->md.M;
+  const bool dense = ctx->md.ablation == TLF_ABLATION_DENSE_CACHE;  // every cache holds a slot per token
   for (int b = 0; b < B; ++b)
-    for (int r = 0; r < ctx->h_m[b]; ++r) ctx->h_len[(size_t)slots[b] * M + r] += 1;
+    for (int r = 0; r < (dense ? M : ctx->h_m[b]); ++r) ctx->h_len[(size_t)slots[b] * M + r] += 1;
 }
 
 // ----------------------------------------------------------------------------
@@ -1222,12 +1231,13 @@ extern "C" int tlf_prefill(tlf_ctx* ctx, int32_t n_seqs, const uint64_t* seq_ids
     return rc;
   };
   const bool logits_dev = last_logits && is_device_ptr(last_logits);
-  if (ctx->use_tc) {  // batched, chunked prefill on the tensor-core path
+  if (ctx->use_tc && ctx->md.ablation != TLF_ABLATION_DENSE_CACHE) {  // batched, chunked prefill (tcgen05)
     const int rc = prefill_batched(ctx, n_seqs, slot_of.data(), offsets, tokens, forced, last_logits, logits_dev,
                                    loops, st);
     return rc ? rollback(rc) : TLF_OK;
   }
-  // float32 models: the prompt runs position by position through the decode kernels
+  // float32 models and the dense-cache ablation: the prompt runs position by position through the
+  // decode kernels
   const int maxB = ctx->cfg.max_batch;
   std::vector<PageUpdate> upd;
   for (int g0 = 0; g0 < n_seqs; g0 += maxB) {
@@ -1300,6 +1310,37 @@ extern "C" int tlf_load_cache(tlf_ctx* ctx, uint64_t seq_id, const int32_t* lens
     }
     need += (lens[r] + ps - 1) / ps;
     off += lens[r];
+  }
+  // without recursion-wise caches (dense-cache ablation) every loop cache holds a slot per position:
+  // slot t of loop r holds position t if the token ran loop r, else a masked slot (position -1)
+  std::vector<int32_t> dlens, dpos;
+  std::vector<uint8_t> hk, hv;
+  if (ctx->md.ablation == TLF_ABLATION_DENSE_CACHE) {
+    const int L0 = lens[0];
+    const size_t ebytes = (size_t)ctx->md.J * ctx->md.Hkv * ctx->md.hd * ctx->eb;
+    dlens.assign(M, L0);
+    dpos.assign((size_t)M * L0, -1);
+    if (!fill) {
+      hk.assign((size_t)M * L0 * ebytes, 0);
+      hv.assign((size_t)M * L0 * ebytes, 0);
+    }
+    for (int r = 0; r < M; ++r)
+      for (int i = 0; i < lens[r]; ++i) {
+        const int t = positions[offs[r] + i];
+        dpos[(size_t)r * L0 + t] = t;
+        if (!fill) {
+          memcpy(&hk[((size_t)r * L0 + t) * ebytes], (const uint8_t*)k + (offs[r] + i) * ebytes, ebytes);
+          memcpy(&hv[((size_t)r * L0 + t) * ebytes], (const uint8_t*)v + (offs[r] + i) * ebytes, ebytes);
+        }
+      }
+    for (int r = 0; r < M; ++r) offs[r] = (size_t)r * L0;
+    lens = dlens.data();
+    positions = dpos.data();
+    if (!fill) {
+      k = hk.data();
+      v = hv.data();
+    }
+    need = (size_t)M * ((L0 + ps - 1) / ps);
   }
   if (need > ctx->free_pages.size()) return fail(ctx, TLF_ERR_OUT_OF_PAGES, "snapshot needs %zu pages", need);
   const int slot = new_slot(ctx, seq_id, 0);

@@ -25,7 +25,7 @@ KERNEL_CLASSES = ("router", "plan", "attn_norm", "qkv_gemm", "rope_append", "att
 DTYPE = {"f32": 0, "bf16": 1}
 EXIT = {"argmax": 0, "survival": 1}
 GEMM = {"auto": 0, "simt": 1}
-ABLATION = {"none": 0, "no_gather": 1}
+ABLATION = {"none": 0, "no_gather": 1, "dense_cache": 2}
 
 
 class TlfConfig(C.Structure):

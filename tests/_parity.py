@@ -72,13 +72,24 @@ def cache_tol(model):
     return 1e-4 if model.dtype == "f32" else 3e-2
 
 
-def check_cache(ctx, seq_id, oseq, model, tol=None):
-    """GPU cache of one sequence against the oracle's: positions exact, K/V within tol."""
+def check_cache(ctx, seq_id, oseq, model, tol=None, masked_slots=False):
+    """GPU cache of one sequence against the oracle's: positions exact, K/V within tol.
+
+    masked_slots: the cache keeps a slot per position (dense-cache ablation); slot t
+    of loop i must hold position t if the token ran loop i, else the mask -1, and
+    the K/V of the unmasked slots are compared.
+    """
     tol = cache_tol(model) if tol is None else tol
     for i in range(model.max_loops):
         for j in range(model.n_layers):
             gp, gk, gv = ctx.read_cache(seq_id, i + 1, j)
             op, ok, ov = oseq.caches[i][j].view()
+            if masked_slots:
+                want = np.full(len(gp), -1, dtype=np.int64)
+                want[np.asarray(op, dtype=np.int64)] = op
+                np.testing.assert_array_equal(gp, want)
+                keep = np.asarray(gp) >= 0
+                gp, gk, gv = gp[keep], gk[keep], gv[keep]
             np.testing.assert_array_equal(gp, op)
             for name, g, o in (("k", gk, ok), ("v", gv, ov)):
                 if not len(op):

@@ -62,10 +62,11 @@ def _greedy_run(T, wl, steps=None, gemm_impl="auto", check_caches=True, ablation
             np.testing.assert_allclose(gmar[free], omar[free], rtol=1e-3, atol=1e-4)
             nxt = np.argmax(olog, axis=1).astype(np.int32)
         if check_caches:
+            dense = ablation == "dense_cache"  # every loop cache has a slot per token
             for b in range(B):
                 for r in range(1, m.max_loops + 1):
-                    assert ctx.cache_len(ids[b], r) == seqs[b].cache_len(r)
-            check_cache(ctx, ids[0], seqs[0], m)
+                    assert ctx.cache_len(ids[b], r) == seqs[b].cache_len(1 if dense else r)
+            check_cache(ctx, ids[0], seqs[0], m, masked_slots=dense)
     return worst, depth.n_forced
 
 
@@ -104,6 +105,8 @@ def _snapshot_run(T, wl, lengths, steps, sampled, seed=7, distinct=2, ablation="
             snaps[key] = synth.make_cache_snapshot(m, int(lengths[b]), seed + 31 * key[1] + int(lengths[b]))
     pages = sum(sum((len(p) + 63) // 64 + 1 for p in snaps[(int(lengths[b]), b % distinct)]["positions"])
                 for b in range(B)) + B * m.max_loops * (steps // 64 + 2)
+    if ablation == "dense_cache":  # every loop cache holds a slot per position
+        pages = B * m.max_loops * ((int(max(lengths)) + steps) // 64 + 2)
     ids = list(range(1000, 1000 + B))
     tokens = synth.make_decode_tokens(wl, steps=steps, batch=B)
     tol = tol_for(m)
@@ -128,13 +131,17 @@ def _snapshot_run(T, wl, lengths, steps, sampled, seed=7, distinct=2, ablation="
                 worst = max(worst, e)
                 assert e < tol, f"step {step} seq {b}: rel err {e}"
         all_loops = np.array(all_loops)
+        dense = ablation == "dense_cache"
         for b in range(B):
             snap = snaps[(int(lengths[b]), b % distinct)]
             for r in range(1, m.max_loops + 1):
-                want = len(snap["positions"][r - 1]) + int((all_loops[:, b] >= r).sum())
+                if dense:
+                    want = len(snap["positions"][0]) + steps
+                else:
+                    want = len(snap["positions"][r - 1]) + int((all_loops[:, b] >= r).sum())
                 assert ctx.cache_len(ids[b], r) == want
         for b in sampled:
-            check_cache(ctx, ids[b], oseqs[b], m)
+            check_cache(ctx, ids[b], oseqs[b], m, masked_slots=dense)
     return worst, depth.n_forced
 
 
@@ -208,7 +215,7 @@ def _prefill_decode_compare(T, m, prompt_lens, steps, forced_mode=None, seed=0, 
             check_active_sets(ctx, gm, m.max_loops, ablation)
             assert rel_err(glog, olog) < tol
         for b in range(B):
-            check_cache(ctx, ids[b], seqs[b], m)
+            check_cache(ctx, ids[b], seqs[b], m, masked_slots=ablation == "dense_cache")
         live, free, total = ctx.stats()
         for i in ids:
             ctx.release(i)
@@ -365,3 +372,22 @@ def test_no_gather_ablation_c5_ragged(tlf):
     worst, forced = _snapshot_run(tlf, wl, lengths, steps=2, sampled=[int(np.argmax(lengths)), int(np.argmin(lengths))],
                                   distinct=1, ablation="no_gather")
     print(f"c5 no-gather worst {worst:.2e} forced {forced}")
+
+
+def test_dense_cache_ablation_c2_greedy(tlf):
+    """Full-length caches read under the mask mu^(r) give the method's results (prefill position by position)."""
+    wl = synth.get_config("c2").with_batch(4)
+    worst, forced = _greedy_run(tlf, wl, steps=12, ablation="dense_cache")
+    print(f"c2 dense-cache worst {worst:.2e} forced {forced}")
+
+
+@pytest.mark.parametrize("lens", [[1, 64, 65], [130, 2, 70, 64]])
+def test_dense_cache_ablation_edges(tlf, lens):
+    _prefill_decode_compare(tlf, _small(), lens, steps=4, ablation="dense_cache")
+
+
+def test_dense_cache_ablation_c3_snapshot(tlf):
+    wl = synth.get_config("c3")
+    lengths = np.full(16, wl.prompt_len[0])
+    worst, forced = _snapshot_run(tlf, wl.with_batch(16), lengths, steps=3, sampled=[0, 5], ablation="dense_cache")
+    print(f"c3 dense-cache worst {worst:.2e} forced {forced}")
