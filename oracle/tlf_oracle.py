@@ -54,6 +54,18 @@ definitions the implementation is built for):
   takes it); everything else is float64.
 * RMSNorm eps = 1e-5 (unstated in the paper).
 * Nothing is written to caches deeper than m (Eq. 11 and the text after it).
+* Time/step conditioning (Sec. 3.1, App. A; only when the weights carry the
+  conditioning MLPs): a token of depth m follows the uniform trajectory of
+  length m, so at loop i it is conditioned on the cumulative time
+  t = c_{i-1} = (i-1)/m and the step Delta = 1/m. Each scalar goes through
+  sinusoidal Fourier features (width 256, max period 10^4; cos and sin of each
+  frequency, in that order) and its own two-layer SiLU MLP; the two results
+  are summed into c. Layer j's modulator maps SiLU(c) linearly to
+  (alpha_msa, alpha_mlp, gamma_msa, gamma_mlp), and the layer computes
+  x <- x + alpha_msa * MHSA(RMSNorm(x) * g * (1 + gamma_msa)) and
+  x <- x + alpha_mlp * FFN(RMSNorm(x) * g * (1 + gamma_mlp)), the gates
+  applied as the equation in App. A writes them (the stored gains g are kept;
+  the paper's norms have none, which gains of one reproduce).
 """
 from __future__ import annotations
 
@@ -67,7 +79,7 @@ __all__ = [
     "rms_norm", "silu", "softmax", "rope", "attention",
     "router_logits", "loop_counts", "decode_token", "decode_step",
     "prefill_sequential", "prefill_gathered", "forward_masked", "load_snapshot",
-    "depth_table",
+    "depth_table", "fourier_features", "trajectory",
 ]
 
 
@@ -84,6 +96,23 @@ def rms_norm(x: np.ndarray, gain: Optional[np.ndarray], eps: float) -> np.ndarra
 
 def silu(x: np.ndarray) -> np.ndarray:
     return x / (1.0 + np.exp(-x))
+
+
+def fourier_features(tau: float, width: int = 256, max_period: float = 10000.0) -> np.ndarray:
+    """[cos(tau w_1), sin(tau w_1), ..., cos(tau w_K), sin(tau w_K)], K = width / 2,
+    w_k = exp(-(k - 1) / K * ln(max_period)) (App. A conditioning embedding)."""
+    K = width // 2
+    w = np.exp(-np.arange(K, dtype=np.float64) / K * np.log(max_period))
+    out = np.empty(width, dtype=np.float64)
+    out[0::2] = np.cos(tau * w)
+    out[1::2] = np.sin(tau * w)
+    return out
+
+
+def trajectory(m: int, i: int) -> Tuple[float, float]:
+    """(cumulative time c_{i-1}, step Delta_i) of loop i for a token of depth m: the uniform
+    trajectory of length m (Sec. 3.1: the full trajectory of L loops has Delta_i = 1/L)."""
+    return (i - 1) / m, 1.0 / m
 
 
 def softmax(z: np.ndarray, axis: int = -1) -> np.ndarray:
@@ -154,10 +183,50 @@ class OracleModel:
                    ffn_hidden=cfg.ffn_hidden, max_loops=cfg.max_loops, rope_base=cfg.rope_base,
                    norm_eps=cfg.norm_eps, exit_rule=cfg.exit_rule, threshold=cfg.threshold, w=w)
 
+    # -- time/step conditioning (Sec. 3.1, App. A) ----------------------------
+    @property
+    def conditioned(self) -> bool:
+        return "mod_w" in self.w
+
+    def phi(self, which: str, tau: float) -> np.ndarray:
+        """Embedding of one scalar: Fourier features, then a two-layer SiLU MLP."""
+        f = fourier_features(tau)
+        hdn = silu(self.w[f"cond_{which}_w1"] @ f + self.w[f"cond_{which}_b1"])
+        return self.w[f"cond_{which}_w2"] @ hdn + self.w[f"cond_{which}_b2"]
+
+    def conditioning(self, m: int, i: int) -> np.ndarray:
+        """c = phi_t(c_{i-1}) + phi_Delta(Delta_i) for a token of depth m at loop i."""
+        t, dt = trajectory(m, i)
+        return self.phi("t", t) + self.phi("dt", dt)
+
+    def modulation(self, j: int, m: int, i: int):
+        """(alpha_msa, alpha_mlp, gamma_msa, gamma_mlp) of layer j, each [d]."""
+        key = (j, m, i)
+        cache = self.__dict__.setdefault("_mod_cache", {})
+        if key not in cache:
+            v = self.w["mod_w"][j] @ silu(self.conditioning(m, i)) + self.w["mod_b"][j]
+            d = self.d_model
+            cache[key] = (v[:d], v[d:2 * d], v[2 * d:3 * d], v[3 * d:])
+        return cache[key]
+
+    def mods(self, j: int, m, i: int):
+        """Per-row modulation for rows of depths m at loop i (None without conditioning).
+
+        Rows with m < i are not run at loop i; they get the vectors of depth i so that
+        vectorised formulations stay finite (their results are discarded).
+        """
+        if not self.conditioned:
+            return None
+        m = np.atleast_1d(np.asarray(m))
+        parts = [self.modulation(j, max(int(mm), i), i) for mm in m]
+        return tuple(np.stack([p[q] for p in parts]) for q in range(4))
+
     # -- pieces of one layer of the shared block --------------------------------
-    def qkv(self, j: int, h: np.ndarray):
+    def qkv(self, j: int, h: np.ndarray, mod=None):
         """Eq. 9: q, k, v of layer j from the incoming states h [..., d]."""
         a = rms_norm(h, self.w["attn_norm"][j], self.norm_eps)
+        if mod is not None:
+            a = a * (1.0 + mod[2].reshape(a.shape))
         q = a @ self.w["wq"][j].T
         k = a @ self.w["wk"][j].T
         v = a @ self.w["wv"][j].T
@@ -166,15 +235,19 @@ class OracleModel:
                 k.reshape(*lead, self.n_kv_heads, self.head_dim),
                 v.reshape(*lead, self.n_kv_heads, self.head_dim))
 
-    def attn_out(self, j: int, o: np.ndarray) -> np.ndarray:
+    def attn_out(self, j: int, o: np.ndarray, mod=None) -> np.ndarray:
         lead = o.shape[:-2]
-        return o.reshape(*lead, self.n_heads * self.head_dim) @ self.w["wo"][j].T
+        y = o.reshape(*lead, self.n_heads * self.head_dim) @ self.w["wo"][j].T
+        return y if mod is None else mod[0].reshape(y.shape) * y
 
-    def mlp(self, j: int, h: np.ndarray) -> np.ndarray:
+    def mlp(self, j: int, h: np.ndarray, mod=None) -> np.ndarray:
         b = rms_norm(h, self.w["mlp_norm"][j], self.norm_eps)
+        if mod is not None:
+            b = b * (1.0 + mod[3].reshape(b.shape))
         g = b @ self.w["w_gate"][j].T
         u = b @ self.w["w_up"][j].T
-        return (silu(g) * u) @ self.w["w_down"][j].T
+        y = (silu(g) * u) @ self.w["w_down"][j].T
+        return y if mod is None else mod[1].reshape(y.shape) * y
 
     def logits(self, h: np.ndarray) -> np.ndarray:
         """Final normalisation and tied LM head on h^(m)."""
@@ -303,15 +376,16 @@ def decode_token(model: OracleModel, seq: OracleSequence, token: int,
     h = model.w["embedding"][token].astype(np.float64)            # h^(0)
     for i in range(1, m + 1):                                      # loops 1..m (early exit after m)
         for j in range(model.n_layers):
-            q, k, v = model.qkv(j, h)                              # Eq. 9
+            mod = model.modulation(j, m, i) if model.conditioned else None
+            q, k, v = model.qkv(j, h, mod)                         # Eq. 9
             q = rope(q, pos, model.rope_base)
             k = rope(k, pos, model.rope_base)
             cache = seq.caches[i - 1][j]
             cache.append(pos, k, v)                                # Eq. 11
             _, kc, vc = cache.view()
             o = attention(q, kc, vc)                               # Eq. 10 (cache i holds only valid entries)
-            h = h + model.attn_out(j, o)
-            h = h + model.mlp(j, h)
+            h = h + model.attn_out(j, o, mod)
+            h = h + model.mlp(j, h, mod)
     seq.n_tokens += 1
     return model.logits(h), m, float(margin[0])
 
@@ -378,7 +452,8 @@ def prefill_gathered(model: OracleModel, seq: OracleSequence, tokens: Sequence[i
             break
         X = H[rho]                                                   # Eq. 6
         for j in range(model.n_layers):
-            q, k, v = model.qkv(j, X)
+            mod = model.mods(j, m[rho], i)
+            q, k, v = model.qkv(j, X, mod)
             q = rope(q, rho[:, None], model.rope_base)
             k = rope(k, rho[:, None], model.rope_base)
             seq.caches[i - 1][j].extend(rho, k, v)                   # written at rho^(i)
@@ -387,8 +462,8 @@ def prefill_gathered(model: OracleModel, seq: OracleSequence, tokens: Sequence[i
                 r1 = min(rho.size, r0 + row_block)
                 allowed = rho[None, :] <= rho[r0:r1, None]
                 o[r0:r1] = _causal_attention(q[r0:r1], k[:r1], v[:r1], allowed[:, :r1])
-            X = X + model.attn_out(j, o)
-            X = X + model.mlp(j, X)
+            X = X + model.attn_out(j, o, mod)
+            X = X + model.mlp(j, X, mod)
         H[rho] = X                                                   # Eq. 7 scatter
     seq.n_tokens = T
     return model.logits(H[-1]), m
@@ -416,7 +491,8 @@ def forward_masked(model: OracleModel, tokens: Sequence[int], m: Sequence[int]) 
             break
         allowed = (pos[None, :] <= pos[:, None]) & mu[None, :]
         for j in range(model.n_layers):
-            q, k, v = model.qkv(j, H)
+            mod = model.mods(j, m, i)
+            q, k, v = model.qkv(j, H, mod)
             q = rope(q, pos[:, None], model.rope_base)
             k = rope(k, pos[:, None], model.rope_base)
             rows = mu.copy()
@@ -424,8 +500,8 @@ def forward_masked(model: OracleModel, tokens: Sequence[int], m: Sequence[int]) 
             safe[~rows] = False
             safe[~rows, 0] = True                                    # rows that are discarded anyway
             o = _causal_attention(q, k, v, safe)
-            Hn = H + model.attn_out(j, o)
-            Hn = Hn + model.mlp(j, Hn)
+            Hn = H + model.attn_out(j, o, mod)
+            Hn = Hn + model.mlp(j, Hn, mod)
             H = np.where(rows[:, None], Hn, H)
     return model.logits(H)
 

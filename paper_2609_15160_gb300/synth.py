@@ -52,6 +52,7 @@ class ModelConfig:
     depth_probs: Optional[Tuple[float, ...]] = None  # target P(m = 1..M); None = no bias
     weight_seed: int = 0
     init_std: float = 0.02
+    conditioning: bool = False     # time/step AdaLN conditioning (Sec. 3.1, App. A)
 
     @property
     def q_dim(self) -> int:
@@ -113,6 +114,9 @@ CONFIGS: Dict[str, WorkloadConfig] = {
                          prompt_seed=3, batch_sweep=(1, 8, 32, 128, 256)),
 }
 CONFIGS["c5f"] = dataclasses.replace(CONFIGS["c5"], name="c5f", forced_loops=8)
+# The C2 and C3 workloads on models with the paper's time/step conditioning (Sec. 3.1, App. A).
+CONFIGS["c2c"] = dataclasses.replace(CONFIGS["c2"], name="c2c", model=dataclasses.replace(_M2, conditioning=True))
+CONFIGS["c3c"] = dataclasses.replace(CONFIGS["c3"], name="c3c", model=dataclasses.replace(_M3, conditioning=True))
 
 
 def get_config(name: str) -> WorkloadConfig:
@@ -225,6 +229,35 @@ def make_weights(m: ModelConfig) -> Dict[str, np.ndarray]:
     w["attn_norm"] = np.ones((J, d), dtype=np.float32)
     w["mlp_norm"] = np.ones((J, d), dtype=np.float32)
     w["final_norm"] = np.ones(d, dtype=np.float32)
+    if m.conditioning:
+        w.update(make_conditioning_weights(m))
+    return w
+
+
+COND_FOURIER = 256  # width of the sinusoidal features of the conditioning scalars (App. A)
+
+
+def make_conditioning_weights(m: ModelConfig) -> Dict[str, np.ndarray]:
+    """Float32 weights of the time/step conditioning (App. A), for each scalar t and dt:
+    cond_{t,dt}_w1 [d, 256], _b1 [d], _w2 [d, d], _b2 [d]; the modulators mod_w [J, 4d, d],
+    mod_b [J, 4d] with outputs ordered (alpha_msa, alpha_mlp, gamma_msa, gamma_mlp).
+
+    The paper zero-initialises the modulator for training; these stand in for trained
+    weights instead: the gate biases are one and the scale biases zero, and the weights
+    are scaled so that the embeddings are of order one and alpha and gamma move by
+    about 0.2 with (t, dt), so that every (depth, loop) pair has its own modulation.
+    """
+    seed, d, J = m.weight_seed, m.d_model, m.n_layers
+    w: Dict[str, np.ndarray] = {}
+    for k, which in enumerate(("t", "dt")):
+        w[f"cond_{which}_w1"] = _normal(seed, 500 + 10 * k, (d, COND_FOURIER), (2.0 / COND_FOURIER) ** 0.5, "f32")
+        w[f"cond_{which}_b1"] = np.zeros(d, dtype=np.float32)
+        w[f"cond_{which}_w2"] = _normal(seed, 501 + 10 * k, (d, d), 1.7 / d ** 0.5, "f32")
+        w[f"cond_{which}_b2"] = np.zeros(d, dtype=np.float32)
+    w["mod_w"] = np.stack([_normal(seed, 600 + j, (4 * d, d), 0.28 / d ** 0.5, "f32") for j in range(J)])
+    b = np.zeros(4 * d, dtype=np.float32)
+    b[:2 * d] = 1.0
+    w["mod_b"] = np.tile(b, (J, 1))
     return w
 
 

@@ -383,12 +383,12 @@ _orig_mlp = O.OracleModel.mlp
 _orig_qkv = O.OracleModel.qkv
 
 
-def _mlp_swapped(self, j, h):
+def _mlp_swapped(self, j, h, mod=None):
     b = O.rms_norm(h, self.w["mlp_norm"][j], self.norm_eps)
     return (O.silu(b @ self.w["w_up"][j].T) * (b @ self.w["w_gate"][j].T)) @ self.w["w_down"][j].T
 
 
-def _qkv_transposed(self, j, h):
+def _qkv_transposed(self, j, h, mod=None):
     a = O.rms_norm(h, self.w["attn_norm"][j], self.norm_eps)
     lead = h.shape[:-1]
     return ((a @ self.w["wq"][j]).reshape(*lead, self.n_heads, self.head_dim),
@@ -396,7 +396,7 @@ def _qkv_transposed(self, j, h):
             (a @ self.w["wv"][j].T).reshape(*lead, self.n_kv_heads, self.head_dim))
 
 
-def _qkv_no_gain(self, j, h):
+def _qkv_no_gain(self, j, h, mod=None):
     a = O.rms_norm(h, None, self.norm_eps)
     lead = h.shape[:-1]
     return ((a @ self.w["wq"][j].T).reshape(*lead, self.n_heads, self.head_dim),
