@@ -41,6 +41,8 @@ DESCR = {
     "c4": "long-context GQA looped LM (d2048 16q/8kv x128 J2 ff5504 M6), batch 16, 32768-token context",
     "c5": "C3 model, ragged prompts U[128,8192], batch 32, routed depths",
     "c5f": "C3 model, ragged prompts U[128,8192], batch 32, every token forced to 8 loops",
+    "c2c": "C2 workload on a model with time/step AdaLN conditioning (Sec. 3.1, App. A)",
+    "c3c": "C3 workload on a model with time/step AdaLN conditioning (Sec. 3.1, App. A)",
 }
 
 

@@ -114,7 +114,11 @@ typedef struct tlf_config {
   int32_t prefill_chunk;/* prompt tokens per batched-prefill chunk (bf16 models); 0 = 8192 */
   int64_t kv_pool_pages;/* pages in the KV pool; 0 = max_seqs * max_loops * ceil(max_seq_len / page_size) */
   int32_t ablation;     /* tlf_ablation; 0 = the method as published */
-  int32_t reserved;     /* must be 0 */
+  int32_t conditioning; /* 0 = none (the workloads' backbone); 1 = time/step AdaLN conditioning
+                         * (Sec. 3.1, App. A), with the cond_* and mod_* weights: a token of depth m
+                         * runs loop i conditioned on t = (i-1)/m and Delta = 1/m; layer j computes
+                         * x += alpha_msa * MHSA(RMSNorm(x) * g * (1 + gamma_msa)) and
+                         * x += alpha_mlp * FFN(RMSNorm(x) * g * (1 + gamma_mlp)) */
 } tlf_config;
 
 /* Host pointers to the weights. Shapes use V, d, Hq, Hkv, hd, J, ff, M from
@@ -134,6 +138,20 @@ typedef struct tlf_weights {
   const float* attn_norm;  /* [J][d] */
   const float* mlp_norm;   /* [J][d] */
   const float* final_norm; /* [d] */
+  /* Time/step conditioning (cfg.conditioning = 1; may be NULL otherwise), float32. For each of the
+   * scalars t and Delta: 256 sinusoidal features [cos(x w_1), sin(x w_1), ...], w_k =
+   * 10000^(-(k-1)/128), then w2 SiLU(w1 f + b1) + b2; c = sum of the two; layer j's modulator
+   * gives mod_w[j] SiLU(c) + mod_b[j] = (alpha_msa, alpha_mlp, gamma_msa, gamma_mlp), d each. */
+  const float* cond_t_w1;  /* [d][256] */
+  const float* cond_t_b1;  /* [d] */
+  const float* cond_t_w2;  /* [d][d] */
+  const float* cond_t_b2;  /* [d] */
+  const float* cond_dt_w1; /* [d][256] */
+  const float* cond_dt_b1; /* [d] */
+  const float* cond_dt_w2; /* [d][d] */
+  const float* cond_dt_b2; /* [d] */
+  const float* mod_w;      /* [J][4d][d] */
+  const float* mod_b;      /* [J][4d] */
 } tlf_weights;
 
 typedef struct tlf_ctx tlf_ctx;

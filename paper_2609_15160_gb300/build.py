@@ -20,7 +20,7 @@ CSRC = os.path.join(PKG, "csrc")
 BUILD = os.path.join(PKG, "_build")
 LIB = os.path.join(BUILD, "libtlf.so")
 INCLUDE = os.path.join(ROOT, "include")
-SOURCES = ["k_router.cu", "k_gemm.cu", "k_attn.cu", "k_misc.cu", "k_prefill.cu", "tlf_api.cu", "tlf_ops.cu",
+SOURCES = ["k_router.cu", "k_gemm.cu", "k_attn.cu", "k_misc.cu", "k_prefill.cu", "k_cond.cu", "tlf_api.cu", "tlf_ops.cu",
            "tlf_static.cu"]
 HEADERS = [os.path.join(CSRC, "tlf_internal.cuh"), os.path.join(INCLUDE, "tlf.h")]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]

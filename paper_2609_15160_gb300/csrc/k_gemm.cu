@@ -39,6 +39,7 @@ __device__ __forceinline__ void gemm_write(const GemmArgs& a, int split, int row
   } else if (a.epi == EPI_RESID) {
     if (a.act && !a.act[row]) return;  // masked row (no-gather ablation): residual unchanged
     const int r = a.idx ? a.idx[row] : row;
+    if (a.alpha.mod) v *= cond_row(a.alpha, r)[col];  // time/step conditioning gate
     atomicAdd(a.resid + (size_t)r * a.ldr + col, v);
   } else {
     a.out[(size_t)row * a.ldo + col] = v;
@@ -111,8 +112,10 @@ __device__ void cluster_epilogue(const GemmArgs& a, float* red, int4* ci, int m0
         cluster_sum4(pb, S, tid, c, c1, sm);
 #pragma unroll
         for (int q = 0; q < 4; ++q)
-          if (c + q < c1)  // the only writer of this element
-            if (ci[c + q].w >= 0) atomicAdd(a.resid + (size_t)ci[c + q].w * a.ldr + col, sm[q]);
+          if (c + q < c1 && ci[c + q].w >= 0) {  // the only writer of this element
+            const float g = a.alpha.mod ? a.alpha.mod[ci[c + q].x + col] : 1.f;
+            atomicAdd(a.resid + (size_t)ci[c + q].w * a.ldr + col, g * sm[q]);
+          }
       }
     return;
   }
@@ -296,9 +299,12 @@ __global__ void __launch_bounds__(128) k_gemm_tc(const __grid_constant__ CUtenso
         if (a.epi == EPI_CL_QKV && !a.row_cslot) {
           colinfo[c] = a.s.rowinfo[a.r * a.md.max_batch + tok0 + c];
         } else if (a.epi == EPI_CL_RESID) {
-          // residual row; -1 for a row masked by the no-gather ablation (residual unchanged)
+          // residual row; -1 for a row masked by the no-gather ablation (residual unchanged);
+          // with time/step conditioning, the offset of the row's gate vector in the table
           const bool masked = a.act && !a.act[tok0 + c];
-          colinfo[c] = make_int4(0, 0, 0, masked ? -1 : (a.idx ? a.idx[tok0 + c] : tok0 + c));
+          const int row = masked ? -1 : (a.idx ? a.idx[tok0 + c] : tok0 + c);
+          const int aoff = (a.alpha.mod && row >= 0) ? (int)(cond_row(a.alpha, row) - a.alpha.mod) : 0;
+          colinfo[c] = make_int4(aoff, 0, 0, row);
         }
       }
     }

@@ -1,7 +1,8 @@
 // Row-wise kernels of the decode step.
 //
 // k_norm_rows    gather + RMSNorm: X[k] = RMSNorm(H[idx[k]]) * gain for the
-//                rows of the active set (Eq. 6 followed by the pre-norm).
+//                rows of the active set (Eq. 6 followed by the pre-norm); with
+//                time/step conditioning the gain is scaled by (1 + gamma).
 // k_rope_table   (cos, sin) of every position x rotary frequency, built once.
 // k_rope_append  sums the split-K partials of the fused QKV projection (Eq. 9),
 //                rotates q and k at the token's original position, keeps q for
@@ -32,7 +33,7 @@ template <typename T>
 __global__ void __launch_bounds__(256) k_norm_rows(const float* __restrict__ H, int ldh, const int* __restrict__ idx,
                                                    const int* __restrict__ n_dev, int n_host,
                                                    const float* __restrict__ gain, int d, float eps,
-                                                   T* __restrict__ X, int ldx) {
+                                                   T* __restrict__ X, int ldx, CondArgs cg) {
   pdl_wait();
   pdl_trigger();
   const int k = blockIdx.x;
@@ -56,11 +57,17 @@ __global__ void __launch_bounds__(256) k_norm_rows(const float* __restrict__ H, 
   ss = block_sum(ss);
   const float inv = rsqrtf(ss / (float)d + eps);
   T* xr = X + (size_t)k * ldx;
+  // time/step conditioning: the gain is scaled by (1 + gamma) of the row's (depth, loop)
+  const float4* c4 = cg.mod ? reinterpret_cast<const float4*>(cond_row(cg, src)) : nullptr;
 #pragma unroll
   for (int c = 0; c < 8; ++c) {
     const int i = threadIdx.x + c * blockDim.x;
     if (i < d4) {
-      const float4 g = g4[i];
+      float4 g = g4[i];
+      if (c4) {
+        const float4 y = c4[i];
+        g = make_float4(g.x * (1.f + y.x), g.y * (1.f + y.y), g.z * (1.f + y.z), g.w * (1.f + y.w));
+      }
       xr[4 * i + 0] = from_f32<T>(v[c].x * inv * g.x);
       xr[4 * i + 1] = from_f32<T>(v[c].y * inv * g.y);
       xr[4 * i + 2] = from_f32<T>(v[c].z * inv * g.z);
@@ -70,12 +77,13 @@ __global__ void __launch_bounds__(256) k_norm_rows(const float* __restrict__ H, 
 }
 
 void launch_norm_rows(int dtype, const float* H, int ldh, const int* idx, const int* n_dev, int n_host, int rows_max,
-                      const float* gain, int d, float eps, void* X, int ldx, cudaStream_t st) {
+                      const float* gain, int d, float eps, void* X, int ldx, cudaStream_t st, const CondArgs& gamma) {
   if (rows_max <= 0) return;
   if (dtype == 1)
-    launch_k(k_norm_rows<bf16>, rows_max, 256, 0, st, H, ldh, idx, n_dev, n_host, gain, d, eps, (bf16*)X, ldx);
+    launch_k(k_norm_rows<bf16>, rows_max, 256, 0, st, H, ldh, idx, n_dev, n_host, gain, d, eps, (bf16*)X, ldx, gamma);
   else
-    launch_k(k_norm_rows<float>, rows_max, 256, 0, st, H, ldh, idx, n_dev, n_host, gain, d, eps, (float*)X, ldx);
+    launch_k(k_norm_rows<float>, rows_max, 256, 0, st, H, ldh, idx, n_dev, n_host, gain, d, eps, (float*)X, ldx,
+             gamma);
 }
 
 // Rotary table: table[p][i] = (cos, sin)(p * theta_i), the angle formed and

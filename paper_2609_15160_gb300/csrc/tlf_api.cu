@@ -64,6 +64,7 @@ struct tlf_ctx {
   float* d_final_norm = nullptr;
   double* d_inv_freq = nullptr;
   float2* d_rope = nullptr;     // [max_pos][hd/2] (cos, sin)
+  float* d_cond = nullptr;      // [J][M(M+1)/2][4][d] time/step modulation (conditioning only)
   int4* d_rowinfo = nullptr;    // [M][max_batch]
   int* d_act = nullptr;         // [M][max_batch]
   std::vector<DeviceMat> wqkv, wo, wgu, wd;
@@ -228,7 +229,7 @@ extern "C" int tlf_validate_config(const tlf_config* c, char* msg, size_t msg_le
     return bad("unknown ablation");
   if (c->ablation == TLF_ABLATION_DENSE_CACHE && c->dtype != TLF_DTYPE_BF16)
     return bad("the dense-cache ablation needs a bf16 model");
-  if (c->reserved != 0) return bad("reserved must be 0");
+  if (c->conditioning != 0 && c->conditioning != 1) return bad("conditioning must be 0 or 1");
   if (msg && msg_len) snprintf(msg, msg_len, "ok");
   return TLF_OK;
 }
@@ -424,6 +425,29 @@ static int create_impl(tlf_ctx* ctx, const tlf_weights* w) {
     CK(ctx, cudaGetLastError());
     CK(ctx, cudaStreamSynchronize(0));
   }
+  if (c.conditioning) {
+    // time/step conditioning: the weights are needed only to build the per-(depth, loop) table
+    const size_t F = 256, dd = (size_t)d * d, J4 = (size_t)J * 4 * d;
+    const float* src[10] = {w->cond_t_w1, w->cond_t_b1, w->cond_t_w2, w->cond_t_b2, w->cond_dt_w1,
+                            w->cond_dt_b1, w->cond_dt_w2, w->cond_dt_b2, w->mod_w, w->mod_b};
+    const size_t cnt[10] = {d * F, (size_t)d, dd, (size_t)d, d * F, (size_t)d, dd, (size_t)d, J4 * d, J4};
+    float* dev[10] = {};
+    rc = 0;
+    for (int i = 0; i < 10 && rc == 0; ++i) {
+      if (!src[i]) rc = fail(ctx, TLF_ERR_BAD_WEIGHTS, "a conditioning weight pointer is NULL");
+      else rc = upload(ctx, (void**)&dev[i], src[i], cnt[i] * 4, "conditioning weights");
+    }
+    const size_t P = (size_t)M * (M + 1) / 2;
+    if (rc == 0) rc = dev_alloc(ctx, &ctx->d_cond, (size_t)J * P * 4 * d * 4, "conditioning table");
+    if (rc == 0) {
+      const int e = build_cond_table(md, dev[0], dev[1], dev[2], dev[3], dev[4], dev[5], dev[6], dev[7], dev[8],
+                                     dev[9], ctx->d_cond, 0);
+      if (e) rc = fail(ctx, TLF_ERR_CUDA, "conditioning table: %s", cudaGetErrorString((cudaError_t)e));
+    }
+    for (float* p : dev)
+      if (p) cudaFree(p);
+    if (rc) return rc;
+  }
 
   // KV pool and tables
   if ((rc = dev_alloc(ctx, &ctx->d_pool, (size_t)ctx->n_pages * page_bytes_of(c), "kv pool"))) return rc;
@@ -517,7 +541,7 @@ extern "C" void tlf_destroy(tlf_ctx* ctx) {
     cudaDeviceSynchronize();
     auto f = [](void* p) { if (p) cudaFree(p); };
     f(ctx->d_emb); f(ctx->d_router_w); f(ctx->d_router_b); f(ctx->d_attn_norm); f(ctx->d_mlp_norm);
-    f(ctx->d_final_norm); f(ctx->d_inv_freq); f(ctx->d_rope); f(ctx->d_rowinfo); f(ctx->d_act);
+    f(ctx->d_final_norm); f(ctx->d_inv_freq); f(ctx->d_rope); f(ctx->d_rowinfo); f(ctx->d_act); f(ctx->d_cond);
     for (auto* v : {&ctx->wqkv, &ctx->wo, &ctx->wgu, &ctx->wd})
       for (auto& m : *v) f(m.ptr);
     f(ctx->d_pool); f(ctx->d_pos_table); f(ctx->d_page_table); f(ctx->d_len); f(ctx->d_upload);
@@ -654,6 +678,21 @@ static void gemm(tlf_ctx* ctx, const DeviceMat& W, const CUtensorMap* xmap, cons
 // buffer, every kernel, and the download of loop counts, margins and the error
 // word. Capturable in a CUDA graph (nothing here depends on host values that
 // change between steps with the same batch size).
+// Lookup of one of the four conditioning vectors (0 alpha_msa, 1 alpha_mlp, 2 gamma_msa,
+// 3 gamma_mlp) of layer j at loop r for rows whose loop counts are m; empty without conditioning.
+static CondArgs cond_args(const tlf_ctx* ctx, const int* m, int r, int j, int part) {
+  CondArgs c;
+  if (!ctx->d_cond) return c;
+  c.mod = ctx->d_cond;
+  c.m = m;
+  c.M = ctx->md.M;
+  c.d = ctx->md.d;
+  c.r = r;
+  c.j = j;
+  c.part = part;
+  return c;
+}
+
 static int enqueue_step(tlf_ctx* ctx, int B, bool need_logits, bool prof, cudaStream_t st) {
   const ModelDims& md = ctx->md;
   const int M = md.M, J = md.J, maxB = md.max_batch;
@@ -703,7 +742,7 @@ static int enqueue_step(tlf_ctx* ctx, int B, bool need_logits, bool prof, cudaSt
     const int* act_r = md.ablation == TLF_ABLATION_NO_GATHER ? ctx->d_act + (size_t)r * maxB : nullptr;
     for (int j = 0; j < J; ++j) {
       launch_norm_rows(md.dtype, ctx->d_H, md.d, idx_r, n_dev, 0, maxB, ctx->d_attn_norm + (size_t)j * md.d, md.d,
-                       md.eps, ctx->d_X, md.d, st);
+                       md.eps, ctx->d_X, md.d, st, cond_args(ctx, s.m, r, j, 2));
       mark(2);
       GemmArgs a{};
       a.n_dev = n_dev;
@@ -739,11 +778,12 @@ static int enqueue_step(tlf_ctx* ctx, int B, bool need_logits, bool prof, cudaSt
       a.ldr = md.d;
       a.idx = idx_r;
       a.act = act_r;
+      a.alpha = cond_args(ctx, s.m, r, j, 0);
       a.splits = ctx->s_o;
       gemm(ctx, ctx->wo[j], &ctx->map_O, ctx->d_O, md.q_dim, a, st);
       mark(6);
       launch_norm_rows(md.dtype, ctx->d_H, md.d, idx_r, n_dev, 0, maxB, ctx->d_mlp_norm + (size_t)j * md.d, md.d,
-                       md.eps, ctx->d_X, md.d, st);
+                       md.eps, ctx->d_X, md.d, st, cond_args(ctx, s.m, r, j, 3));
       mark(7);
       a = GemmArgs{};
       a.n_dev = n_dev;
@@ -772,6 +812,7 @@ static int enqueue_step(tlf_ctx* ctx, int B, bool need_logits, bool prof, cudaSt
       a.ldr = md.d;
       a.idx = idx_r;
       a.act = act_r;
+      a.alpha = cond_args(ctx, s.m, r, j, 1);
       a.splits = ctx->s_d;
       gemm(ctx, ctx->wd[j], &ctx->map_U, ctx->d_U, md.ff, a, st);
       mark(10);
@@ -1107,7 +1148,7 @@ static int prefill_batched(tlf_ctx* ctx, int n_seqs, const int* slot_of, const i
       const int* idx_r = ctx->d_pf_idx + (size_t)r * C;
       for (int j = 0; j < J; ++j) {
         launch_norm_rows(md.dtype, ctx->d_pf_H, md.d, idx_r, n_dev, 0, C, ctx->d_attn_norm + (size_t)j * md.d, md.d,
-                         md.eps, ctx->d_pf_X, md.d, st);
+                         md.eps, ctx->d_pf_X, md.d, st, cond_args(ctx, ctx->d_pf_m, r, j, 2));
         GemmArgs a{};
         a.n_dev = n_dev;
         a.epi = EPI_CL_QKV;
@@ -1128,9 +1169,10 @@ static int prefill_batched(tlf_ctx* ctx, int n_seqs, const int* slot_of, const i
         a.resid = ctx->d_pf_H;
         a.ldr = md.d;
         a.idx = idx_r;
+        a.alpha = cond_args(ctx, ctx->d_pf_m, r, j, 0);
         gemm_pf(ctx, ctx->wo[j], &ctx->pf_map_O, a, st);
         launch_norm_rows(md.dtype, ctx->d_pf_H, md.d, idx_r, n_dev, 0, C, ctx->d_mlp_norm + (size_t)j * md.d, md.d,
-                         md.eps, ctx->d_pf_X, md.d, st);
+                         md.eps, ctx->d_pf_X, md.d, st, cond_args(ctx, ctx->d_pf_m, r, j, 3));
         a = GemmArgs{};
         a.n_dev = n_dev;
         a.epi = EPI_CL_SWIGLU;
@@ -1143,6 +1185,7 @@ static int prefill_batched(tlf_ctx* ctx, int n_seqs, const int* slot_of, const i
         a.resid = ctx->d_pf_H;
         a.ldr = md.d;
         a.idx = idx_r;
+        a.alpha = cond_args(ctx, ctx->d_pf_m, r, j, 1);
         gemm_pf(ctx, ctx->wd[j], &ctx->pf_map_U, a, st);
       }
     }

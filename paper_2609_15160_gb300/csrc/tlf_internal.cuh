@@ -337,12 +337,32 @@ struct ModelDims {
   int ablation;          // tlf_ablation
 };
 
+// Time/step conditioning (Sec. 3.1, App. A) inside the step. The modulation of
+// layer j for a token of depth m at loop r (0-based) is built once per context
+// into the table [J][M(M+1)/2][4][d]: depth-major (m, r) pairs, then the four
+// vectors alpha_msa, alpha_mlp, gamma_msa, gamma_mlp.
+struct CondArgs {
+  const float* mod = nullptr;  // the table; NULL = no conditioning
+  const int* m = nullptr;      // loop count of each row, indexed like the residual stream's rows
+  int M = 0, d = 0, r = 0, j = 0;
+  int part = 0;                // which of the four vectors
+};
+// Row of the table for residual-stream row b. Rows that do not run loop r (masked
+// rows of the no-gather ablation, discarded) read the vectors of depth r + 1.
+__device__ __forceinline__ const float* cond_row(const CondArgs& c, int b) {
+  int m = c.m[b];
+  m = m < c.r + 1 ? c.r + 1 : (m > c.M ? c.M : m);
+  const int combo = m * (m - 1) / 2 + c.r;
+  return c.mod + (((size_t)c.j * (c.M * (c.M + 1) / 2) + combo) * 4 + c.part) * c.d;
+}
+
 struct GemmArgs {
   int N;             // output features (rows of W)
   int K;             // reduction length
   int splits;        // split-K factor (gridDim.y; the cluster size for EPI_CL_*)
   int stages;        // depth of the tcgen05 kernel's operand ring (set by the launcher)
   const int* act;    // RESID epilogues: rows with act[row] == 0 keep their residual (NULL: none)
+  CondArgs alpha;    // RESID epilogues: the update is gated by alpha (conditioning; mod NULL: none)
   const int* n_dev;  // token rows n (device scalar), or NULL to use n_host
   int n_host;
   int epi;           // GemmEpilogue
@@ -381,7 +401,12 @@ void launch_router(const ModelDims& md, const StepDev& s, int B, const void* emb
 void launch_plan(const ModelDims& md, const StepDev& s, int B, cudaStream_t st);
 
 void launch_norm_rows(int dtype, const float* H, int ldh, const int* idx, const int* n_dev, int n_host,
-                      int rows_max, const float* gain, int d, float eps, void* X, int ldx, cudaStream_t st);
+                      int rows_max, const float* gain, int d, float eps, void* X, int ldx, cudaStream_t st,
+                      const CondArgs& gamma = CondArgs{});
+// Builds the conditioning table (see CondArgs) from the float32 weights on the device, in float64.
+int build_cond_table(const ModelDims& md, const float* t_w1, const float* t_b1, const float* t_w2, const float* t_b2,
+                     const float* dt_w1, const float* dt_b1, const float* dt_w2, const float* dt_b2,
+                     const float* mod_w, const float* mod_b, float* table, cudaStream_t st);
 
 void launch_gemm_simt(int dtype, const void* W, const void* X, int ldx, const GemmArgs& a, cudaStream_t st);
 void launch_gemm_tc(const CUtensorMap* mapW, const CUtensorMap* mapX, int nt_max, const GemmArgs& a,

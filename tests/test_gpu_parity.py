@@ -391,3 +391,29 @@ def test_dense_cache_ablation_c3_snapshot(tlf):
     lengths = np.full(16, wl.prompt_len[0])
     worst, forced = _snapshot_run(tlf, wl.with_batch(16), lengths, steps=3, sampled=[0, 5], ablation="dense_cache")
     print(f"c3 dense-cache worst {worst:.2e} forced {forced}")
+
+
+# ----------------------------------------------------------------------------
+# time/step AdaLN conditioning (Sec. 3.1, App. A)
+# ----------------------------------------------------------------------------
+
+def test_conditioning_c2c_greedy(tlf):
+    """Per-token (depth, loop) modulation applied in the norms and residual gates, prefill and decode."""
+    worst, forced = _greedy_run(tlf, synth.get_config("c2c"), steps=24)
+    print(f"c2c worst {worst:.2e} forced {forced}")
+
+
+def test_conditioning_c3c_full_size_sampled(tlf):
+    wl = synth.get_config("c3c")
+    lengths = np.full(wl.batch, wl.prompt_len[0])
+    worst, forced = _snapshot_run(tlf, wl, lengths, steps=3, sampled=[0, 41])
+    print(f"c3c worst {worst:.2e} forced {forced}")
+
+
+@pytest.mark.parametrize("dtype,gemm_impl", [("bf16", "auto"), ("bf16", "simt"), ("f32", "auto")])
+def test_conditioning_small_models(tlf, dtype, gemm_impl):
+    _prefill_decode_compare(tlf, _small(dtype, conditioning=True), [70, 1, 130], steps=4, gemm_impl=gemm_impl)
+
+
+def test_conditioning_with_no_gather(tlf):
+    _prefill_decode_compare(tlf, _small(conditioning=True), [65, 3, 64], steps=3, ablation="no_gather")

@@ -49,7 +49,7 @@ def _cfg(**kw):
 @pytest.mark.parametrize("field,value", [
     ("d_model", 100), ("n_kv_heads", 3), ("head_dim", 48), ("max_loops", 0), ("max_loops", 17),
     ("max_batch", 0), ("max_batch", 300), ("page_size", 32), ("dtype", 7), ("ffn_hidden", 1000),
-    ("exit_rule", 5), ("norm_eps", 0.0), ("max_seqs", 2), ("ablation", 9), ("reserved", 1),
+    ("exit_rule", 5), ("norm_eps", 0.0), ("max_seqs", 2), ("ablation", 9), ("conditioning", 2),
 ])
 def test_validate_config_rejects(lib, field, value):
     rc, msg = tlf.tlf_validate_config(_cfg(**{field: value}))
