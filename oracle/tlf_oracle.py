@@ -43,7 +43,10 @@ definitions the implementation is built for):
   every entry of that cache, itself included (Eq. 10 writes K_{<t}, Eq. 11
   appends k_t; the softmax set is never empty).
 * Router input: RMSNorm (no gain) of h^(0) = E[x] followed by a linear map
-  with bias, d -> M. (The paper's router is a two-layer MLP on E + E_pos; the
+  with bias, d -> M; or, with router weights router_w1 / router_b1, the
+  paper's two-layer MLP: a hidden layer of width H_r with the exact GELU (the
+  activation of the paper's block MLP; the router's own is unstated), then
+  the linear map H_r -> M. (The paper's router is a two-layer MLP on E + E_pos; the
   workloads use RoPE, so the router sees only the token embedding and the
   loop count is a function of the token id.)
 * Exit rule "argmax": m = 1 + argmax_l z_l, ties to the smaller depth,
@@ -79,7 +82,7 @@ __all__ = [
     "rms_norm", "silu", "softmax", "rope", "attention",
     "router_logits", "loop_counts", "decode_token", "decode_step",
     "prefill_sequential", "prefill_gathered", "forward_masked", "load_snapshot",
-    "depth_table", "fourier_features", "trajectory",
+    "depth_table", "fourier_features", "trajectory", "gelu",
 ]
 
 
@@ -96,6 +99,12 @@ def rms_norm(x: np.ndarray, gain: Optional[np.ndarray], eps: float) -> np.ndarra
 
 def silu(x: np.ndarray) -> np.ndarray:
     return x / (1.0 + np.exp(-x))
+
+
+def gelu(x: np.ndarray) -> np.ndarray:
+    """x * Phi(x), Phi the standard normal CDF (the exact GELU)."""
+    from scipy.special import erf
+    return 0.5 * x * (1.0 + erf(x / np.sqrt(2.0)))
 
 
 def fourier_features(tau: float, width: int = 256, max_period: float = 10000.0) -> np.ndarray:
@@ -259,9 +268,15 @@ class OracleModel:
 # ----------------------------------------------------------------------------
 
 def router_logits(model: OracleModel, tokens) -> np.ndarray:
-    """z = W_r RMSNorm(h^(0)) + b_r with h^(0) = E[x]; returns [n, M] float64."""
+    """z = W_r RMSNorm(h^(0)) + b_r with h^(0) = E[x]; returns [n, M] float64.
+
+    With the two-layer MLP router of Sec. 3.2 (weights router_w1 [H_r, d], router_b1 [H_r]):
+    z = W_r GELU(W_1 RMSNorm(h^(0)) + b_1) + b_r, router_w then [M, H_r].
+    """
     h0 = model.w["embedding"][np.asarray(tokens, dtype=np.int64)]
     x = rms_norm(h0, None, model.norm_eps)
+    if "router_w1" in model.w:
+        x = gelu(x @ model.w["router_w1"].T + model.w["router_b1"])
     return x @ model.w["router_w"].T + model.w["router_b"]
 
 

@@ -53,6 +53,7 @@ class ModelConfig:
     weight_seed: int = 0
     init_std: float = 0.02
     conditioning: bool = False     # time/step AdaLN conditioning (Sec. 3.1, App. A)
+    router_hidden: int = 0         # > 0: the two-layer MLP router of Sec. 3.2 with this hidden width
 
     @property
     def q_dim(self) -> int:
@@ -215,11 +216,20 @@ def make_weights(m: ModelConfig) -> Dict[str, np.ndarray]:
     d, J = m.d_model, m.n_layers
     w: Dict[str, np.ndarray] = {}
     w["embedding"] = _normal(seed, 0, (m.vocab, d), std, dt)
-    w["router_w"] = _normal(seed, 1, (m.max_loops, d), std, dt)
-    if m.depth_probs is None:
+    if m.router_hidden > 0:
+        # two-layer MLP router: hidden pre-activations of order one, logits spread over a few units
+        # so that the depth decisions are well separated; no bias fit (the distribution is whatever
+        # these seeded weights give)
+        w["router_w1"] = _normal(seed, 2, (m.router_hidden, d), 1.0 / d ** 0.5, dt)
+        w["router_b1"] = _normal(seed, 3, (m.router_hidden,), 0.5, "f32")
+        w["router_w"] = _normal(seed, 1, (m.max_loops, m.router_hidden), 3.0 / m.router_hidden ** 0.5, dt)
         w["router_b"] = np.zeros(m.max_loops, dtype=np.float32)
     else:
-        w["router_b"] = calibrate_router_bias(w["router_w"], m.depth_probs, std, m.norm_eps, seed)
+        w["router_w"] = _normal(seed, 1, (m.max_loops, d), std, dt)
+        if m.depth_probs is None:
+            w["router_b"] = np.zeros(m.max_loops, dtype=np.float32)
+        else:
+            w["router_b"] = calibrate_router_bias(w["router_w"], m.depth_probs, std, m.norm_eps, seed)
     shapes = {
         "wq": (m.q_dim, d), "wk": (m.kv_dim, d), "wv": (m.kv_dim, d), "wo": (d, m.q_dim),
         "w_gate": (m.ffn_hidden, d), "w_up": (m.ffn_hidden, d), "w_down": (d, m.ffn_hidden),

@@ -191,6 +191,40 @@ def test_survival_rule_nesting_and_median():
     assert m.min() >= 1 and m.max() <= 6
 
 
+def _mlp_router_model(d=16, hidden=24, M=4, seed=9):
+    cfg = synth.tiny_config(router_hidden=hidden, max_loops=M)
+    return cfg, synth.make_weights(cfg)
+
+
+def test_gelu_matches_torch():
+    x = np.linspace(-8, 8, 401)
+    np.testing.assert_allclose(O.gelu(x), F.gelu(torch.tensor(x), approximate="none").numpy(), rtol=1e-14, atol=1e-15)
+
+
+def test_mlp_router_matches_torch():
+    """The two-layer MLP router (Sec. 3.2) against torch library routines."""
+    cfg, w = _mlp_router_model()
+    model = O.OracleModel.from_config(cfg, w)
+    toks = np.arange(cfg.vocab)
+    t = lambda a: torch.tensor(np.asarray(a, dtype=np.float64))
+    x = F.rms_norm(t(w["embedding"])[torch.as_tensor(toks)], (cfg.d_model,), eps=cfg.norm_eps)
+    z = F.linear(F.gelu(F.linear(x, t(w["router_w1"]), t(w["router_b1"]))), t(w["router_w"]), t(w["router_b"]))
+    np.testing.assert_allclose(O.router_logits(model, toks), z.numpy(), rtol=1e-12, atol=1e-12)
+
+
+def test_mlp_router_reduces_to_the_linear_router():
+    """W_1 = I and a large b_1 make GELU the identity shifted by b_1: the linear router with bias b_r + b_1 W_r 1."""
+    cfg, w = _mlp_router_model(hidden=16)
+    d = cfg.d_model
+    wm = dict(w, router_w1=np.eye(d), router_b1=np.full(d, 40.0))
+    lin = {k: v for k, v in w.items() if k not in ("router_w1", "router_b1")}
+    lin["router_b"] = w["router_b"].astype(np.float64) + 40.0 * w["router_w"].astype(np.float64).sum(axis=1)
+    toks = np.arange(cfg.vocab)
+    z_mlp = O.router_logits(O.OracleModel.from_config(cfg, wm), toks)
+    z_lin = O.router_logits(O.OracleModel.from_config(cfg, lin), toks)
+    np.testing.assert_allclose(z_mlp, z_lin, rtol=1e-12, atol=1e-10)
+
+
 def test_router_reads_only_the_embedding():
     """The loop count is a function of the token id (R2 reading)."""
     cfg, w, model, toks = _tiny(max_loops=4)
@@ -444,6 +478,18 @@ def _decode_shared_cache(model, seq, token, forced=None):
     return model.logits(h), m, 0.0
 
 
+def _gelu_tanh(x):
+    return 0.5 * x * (1.0 + np.tanh(np.sqrt(2.0 / np.pi) * (x + 0.044715 * x ** 3)))
+
+
+def _router_no_hidden_bias(model, tokens):
+    h0 = model.w["embedding"][np.asarray(tokens, dtype=np.int64)]
+    x = O.rms_norm(h0, None, model.norm_eps)
+    if "router_w1" in model.w:
+        x = O.gelu(x @ model.w["router_w1"].T)
+    return x @ model.w["router_w"].T + model.w["router_b"]
+
+
 def _loop_counts_off_by_one(model, z):
     m, g = _orig_loop_counts(model, z)
     return np.minimum(m + 1, model.max_loops).astype(np.int32), g
@@ -477,6 +523,8 @@ PLANTS = {
     "shared_cache": ("decode_token", _decode_shared_cache),
     "depth_off_by_one": ("loop_counts", _loop_counts_off_by_one),
     "threshold_ge": ("loop_counts", _loop_counts_ge),
+    "gelu_tanh": ("gelu", _gelu_tanh),
+    "router_hidden_bias_dropped": ("router_logits", _router_no_hidden_bias),
 }
 
 
@@ -488,6 +536,9 @@ def _all_pins_pass():
         test_routed_prefill_uses_router_depths,
         test_cache_content_invariant,
         test_exited_token_leaves_deeper_caches_untouched,
+        test_gelu_matches_torch,
+        test_mlp_router_matches_torch,
+        test_mlp_router_reduces_to_the_linear_router,
     ]
     for t in tests:
         try:
