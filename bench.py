@@ -437,6 +437,63 @@ def run_attn_op(args):
                                    "algorithmic_bytes_per_call": kv_bytes + io_bytes}}))
 
 
+def run_sweep(args):
+    """Decode throughput and mean depth under the SURVIVAL rule of Eq. 4 at several thresholds.
+
+    The paper sweeps the router threshold (Fig. 4c: perplexity and average depth); here the
+    workload's model is rebuilt with exit_rule = survival at each threshold (optionally with the
+    two-layer MLP router), its prompts are prefilled through the library (so the cached tokens carry
+    that threshold's routing too), and decode steps are timed with CUDA events. The ARGMAX rule of
+    the workload is the first row.
+    """
+    import dataclasses
+
+    import torch
+
+    from paper_2609_15160_gb300 import tlf as T
+
+    T.load_library()
+    wl0 = synth.get_config(args.config)
+    rows = []
+    variants = [("argmax", None)] + [("survival", float(t)) for t in args.thresholds.split(",")]
+    for rule, th in variants:
+        m = dataclasses.replace(wl0.model, exit_rule=rule, threshold=th if th is not None else 0.5,
+                                router_hidden=args.router_hidden)
+        wl = dataclasses.replace(wl0, model=m)
+        t0 = time.time()
+        ctx, ids, how = setup_workload(T, wl, 0, prefill=args.prefill, extra_tokens=args.warmup + args.steps + 2)
+        setup_s = time.time() - t0
+        B = wl.batch
+        toks = synth.make_decode_tokens(wl, steps=args.warmup + args.steps, batch=B)
+        logits = torch.empty((B, m.vocab), dtype=torch.float32, device="cuda")
+        st = torch.cuda.current_stream()
+        for k in range(args.warmup):
+            ctx.decode_step(ids, toks[k], logits=logits, stream=st)
+        torch.cuda.synchronize()
+        ev = [torch.cuda.Event(enable_timing=True) for _ in range(2)]
+        loops = []
+        ev[0].record(st)
+        for k in range(args.steps):
+            _, lp, _ = ctx.decode_step(ids, toks[args.warmup + k], logits=logits, stream=st)
+            loops.append(lp)
+        ev[1].record(st)
+        torch.cuda.synchronize()
+        ms = ev[0].elapsed_time(ev[1]) / args.steps
+        lp = np.concatenate(loops)
+        rows.append({"exit_rule": rule, "threshold": th, "ms_per_step": ms, "tokens_per_s": B / (ms * 1e-3),
+                     "mean_loops": float(lp.mean()),
+                     "depth_histogram": np.bincount(lp, minlength=m.max_loops + 1)[1:].tolist(),
+                     "cache": how, "setup_s": setup_s})
+        ctx.close()
+    print(json.dumps({"metric": "decode_tokens_per_s_vs_router_threshold", "unit": "tokens/s",
+                      "higher_is_better": True, "steps": args.steps, "warmup": args.warmup, "dtype": wl0.model.dtype,
+                      "data": "synthetic",
+                      "config": {"workload": DESCR[args.config], "name": args.config,
+                                 "router": f"two-layer MLP, hidden {args.router_hidden}" if args.router_hidden
+                                 else "linear"},
+                      "sweep": rows}))
+
+
 def run_ttft(args):
     """Time to first token: one prompt of each length through tlf_prefill (logits of its last token).
 
@@ -488,8 +545,12 @@ def run_ttft(args):
 
 def main():
     ap = argparse.ArgumentParser()
-    ap.add_argument("--op", default=None, choices=["attn", "ttft"],
-                    help="time one operation alone: the attention kernels, or prefill (time to first token)")
+    ap.add_argument("--op", default=None, choices=["attn", "ttft", "sweep"],
+                    help="time one operation alone: the attention kernels, prefill (time to first token), "
+                         "or decode under the survival rule at several thresholds")
+    ap.add_argument("--thresholds", default="0.2,0.3,0.4,0.5,0.6,0.7,0.8", help="--op sweep: survival thresholds")
+    ap.add_argument("--router-hidden", type=int, default=0,
+                    help="--op sweep: hidden width of the two-layer MLP router (0 = the workload's linear router)")
     ap.add_argument("--ttft-lengths", default="128,512,1024,2048")
     ap.add_argument("--full", action="store_true", help="--op ttft: also prefill the workload's whole batch")
     ap.add_argument("--batch", type=int, default=16)
@@ -517,6 +578,8 @@ def main():
         run_attn_op(args)
     elif args.op == "ttft":
         run_ttft(args)
+    elif args.op == "sweep":
+        run_sweep(args)
     elif args.impl == "reference":
         run_reference(args)
     else:

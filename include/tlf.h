@@ -119,6 +119,10 @@ typedef struct tlf_config {
                          * runs loop i conditioned on t = (i-1)/m and Delta = 1/m; layer j computes
                          * x += alpha_msa * MHSA(RMSNorm(x) * g * (1 + gamma_msa)) and
                          * x += alpha_mlp * FFN(RMSNorm(x) * g * (1 + gamma_mlp)) */
+  int32_t router_hidden;/* 0 = linear router d -> M (the workloads); H_r > 0 (multiple of 8, <= 8192) = the
+                         * two-layer MLP router of Sec. 3.2: z = W_r GELU(W_1 RMSNorm(h0) + b_1) + b_r
+                         * with the exact GELU, weights router_w1/router_b1, router_w then [M][H_r] */
+  int32_t reserved;     /* must be 0 */
 } tlf_config;
 
 /* Host pointers to the weights. Shapes use V, d, Hq, Hkv, hd, J, ff, M from
@@ -126,7 +130,7 @@ typedef struct tlf_config {
  * is in the config dtype. The library copies them to the GPU in tlf_create. */
 typedef struct tlf_weights {
   const void* embedding;   /* [V][d] */
-  const void* router_w;    /* [M][d] */
+  const void* router_w;    /* [M][d], or [M][H_r] with the MLP router */
   const float* router_b;   /* [M] */
   const void* wq;          /* [J][Hq*hd][d] */
   const void* wk;          /* [J][Hkv*hd][d] */
@@ -152,6 +156,8 @@ typedef struct tlf_weights {
   const float* cond_dt_b2; /* [d] */
   const float* mod_w;      /* [J][4d][d] */
   const float* mod_b;      /* [J][4d] */
+  const void* router_w1;   /* [H_r][d] (cfg.router_hidden > 0; may be NULL otherwise) */
+  const float* router_b1;  /* [H_r] */
 } tlf_weights;
 
 typedef struct tlf_ctx tlf_ctx;

@@ -17,6 +17,53 @@
 
 namespace tlf {
 
+// Loop count from the M router logits z (entries >= M are ignored): the ARGMAX or
+// SURVIVAL rule of Eq. 2-5 (see tlf.h), with the decision margin.
+__device__ __forceinline__ void router_decide(const ModelDims& md, const float z[16], int& m, float& margin) {
+  const int M = md.M;
+  m = 1;
+  if (md.exit_rule == 0) {
+    // ARGMAX: first maximum wins (ties go to the smaller depth)
+    int top = 0;
+#pragma unroll
+    for (int l = 1; l < 16; ++l)
+      if (l < M && z[l] > z[top]) top = l;
+    float second = -INFINITY;
+#pragma unroll
+    for (int l = 0; l < 16; ++l)
+      if (l < M && l != top) second = fmaxf(second, z[l]);
+    m = top + 1;
+    margin = z[top] - second;  // +inf when M == 1
+  } else {
+    // SURVIVAL (Eq. 2-5): softmax, suffix sums p^(i), m = max{i : p^(i) > threshold}
+    float mx = z[0];
+#pragma unroll
+    for (int l = 1; l < 16; ++l)
+      if (l < M) mx = fmaxf(mx, z[l]);
+    float ex[16], sum = 0.f;
+#pragma unroll
+    for (int l = 0; l < 16; ++l) {
+      ex[l] = (l < M) ? expf(z[l] - mx) : 0.f;
+      sum += ex[l];
+    }
+    float p[17];
+    p[16] = 0.f;
+    float acc = 0.f;
+#pragma unroll
+    for (int l = 15; l >= 0; --l) {
+      acc += ex[l] / sum;
+      p[l] = acc;
+    }
+    m = 1;
+#pragma unroll
+    for (int l = 0; l < 16; ++l)
+      if (l < M && p[l] > md.threshold) m = l + 1;
+    const float pm = p[m - 1];
+    const float pnext = (m < M) ? p[m] : 0.f;
+    margin = fminf(pm - md.threshold, md.threshold - pnext);
+  }
+}
+
 template <typename T>
 __global__ void __launch_bounds__(256) k_router(ModelDims md, StepDev s, int B, const T* __restrict__ emb,
                                                 const T* __restrict__ rw, const float* __restrict__ rb,
@@ -71,51 +118,103 @@ __global__ void __launch_bounds__(256) k_router(ModelDims md, StepDev s, int B, 
 #pragma unroll
   for (int l = 0; l < 16; ++l) z[l] = (l < M) ? warp_sum(dot[l]) * inv + rb[l] : -INFINITY;
 
-  int m = 1;
+  int m;
   float margin;
-  if (md.exit_rule == 0) {
-    // ARGMAX: first maximum wins (ties go to the smaller depth)
-    int top = 0;
-#pragma unroll
-    for (int l = 1; l < 16; ++l)
-      if (l < M && z[l] > z[top]) top = l;
-    float second = -INFINITY;
-#pragma unroll
-    for (int l = 0; l < 16; ++l)
-      if (l < M && l != top) second = fmaxf(second, z[l]);
-    m = top + 1;
-    margin = z[top] - second;  // +inf when M == 1
-  } else {
-    // SURVIVAL (Eq. 2-5): softmax, suffix sums p^(i), m = max{i : p^(i) > threshold}
-    float mx = z[0];
-#pragma unroll
-    for (int l = 1; l < 16; ++l)
-      if (l < M) mx = fmaxf(mx, z[l]);
-    float ex[16], sum = 0.f;
-#pragma unroll
-    for (int l = 0; l < 16; ++l) {
-      ex[l] = (l < M) ? expf(z[l] - mx) : 0.f;
-      sum += ex[l];
-    }
-    float p[17];
-    p[16] = 0.f;
-    float acc = 0.f;
-#pragma unroll
-    for (int l = 15; l >= 0; --l) {
-      acc += ex[l] / sum;
-      p[l] = acc;
-    }
-    m = 1;
-#pragma unroll
-    for (int l = 0; l < 16; ++l)
-      if (l < M && p[l] > md.threshold) m = l + 1;
-    const float pm = p[m - 1];
-    const float pnext = (m < M) ? p[m] : 0.f;
-    margin = fminf(pm - md.threshold, md.threshold - pnext);
-  }
+  router_decide(md, z, m, margin);
   const int f = s.forced[b];
   if (f >= 1) m = min(f, M);
   if (lane == 0) {
+    s.m[b] = m;
+    s.margin[b] = margin;
+  }
+}
+
+// The two-layer MLP router of Sec. 3.2: z = W_r GELU(W_1 RMSNorm(h0) + b_1) + b_r (exact GELU).
+// One CTA per token: the embedding row goes to the residual stream and, unnormalised, to shared
+// memory; a warp per hidden unit reads its W_1 row in 16-byte chunks (the RMSNorm scale, a
+// per-token scalar, multiplies the dot product), then a warp per logit reads W_r.
+template <typename T>
+__global__ void __launch_bounds__(256) k_router_mlp(ModelDims md, StepDev s, int B, const T* __restrict__ emb,
+                                                    const T* __restrict__ w1, const float* __restrict__ b1,
+                                                    const T* __restrict__ rw, const float* __restrict__ rb,
+                                                    const PageUpdate* __restrict__ upd,
+                                                    const int* __restrict__ n_upd_dev) {
+  pdl_wait();
+  pdl_trigger();
+  const int n_upd = *n_upd_dev;
+  for (int u = blockIdx.x * blockDim.x + threadIdx.x; u < n_upd; u += gridDim.x * blockDim.x) {
+    const PageUpdate p = upd[u];
+    s.page_table[p.index] = p.page;
+  }
+  const int b = blockIdx.x;
+  if (b >= B) return;
+  extern __shared__ float rsm[];
+  const int d = md.d, Hr = md.router_hidden, M = md.M;
+  float* xs = rsm;           // [d]  h0
+  float* hs = rsm + d;       // [Hr] hidden activations
+  __shared__ float zs[16], red[8];
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  int tok = s.tokens[b];
+  if (tok < 0 || tok >= md.V) {
+    if (threadIdx.x == 0) atomicOr(s.err, DEVERR_INDEX);
+    tok = 0;
+  }
+  constexpr int VEC = Vec16<T>::N;
+  const T* e = emb + (size_t)tok * d;
+  float* h = s.H + (size_t)b * d;
+  float ss = 0.f;
+  for (int c = threadIdx.x; c < d / VEC; c += blockDim.x) {
+    float x[VEC];
+    Vec16<T>::load(e + c * VEC, x);
+#pragma unroll
+    for (int u = 0; u < VEC; ++u) {
+      xs[c * VEC + u] = x[u];
+      h[c * VEC + u] = x[u];
+      ss = fmaf(x[u], x[u], ss);
+    }
+  }
+  ss = warp_sum(ss);
+  if (lane == 0) red[warp] = ss;
+  __syncthreads();
+  float tot = 0.f;
+#pragma unroll
+  for (int w = 0; w < 8; ++w) tot += red[w];
+  const float inv = rsqrtf(tot / (float)d + md.eps);
+  for (int u = warp; u < Hr; u += 8) {
+    const T* wr = w1 + (size_t)u * d;
+    float acc = 0.f;
+    for (int c = lane; c < d / VEC; c += 32) {
+      float wv[VEC];
+      Vec16<T>::load(wr + c * VEC, wv);
+#pragma unroll
+      for (int q = 0; q < VEC; ++q) acc = fmaf(wv[q], xs[c * VEC + q], acc);
+    }
+    acc = warp_sum(acc) * inv + b1[u];
+    if (lane == 0) hs[u] = 0.5f * acc * (1.f + erff(acc * 0.70710678118654752f));
+  }
+  __syncthreads();
+  for (int l = warp; l < M; l += 8) {
+    const T* wr = rw + (size_t)l * Hr;
+    float acc = 0.f;
+    for (int c = lane; c < Hr / VEC; c += 32) {
+      float wv[VEC];
+      Vec16<T>::load(wr + c * VEC, wv);
+#pragma unroll
+      for (int q = 0; q < VEC; ++q) acc = fmaf(wv[q], hs[c * VEC + q], acc);
+    }
+    acc = warp_sum(acc);
+    if (lane == 0) zs[l] = acc + rb[l];
+  }
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    float z[16];
+#pragma unroll
+    for (int l = 0; l < 16; ++l) z[l] = (l < M) ? zs[l] : -INFINITY;
+    int m;
+    float margin;
+    router_decide(md, z, m, margin);
+    const int f = s.forced[b];
+    if (f >= 1) m = min(f, M);
     s.m[b] = m;
     s.margin[b] = margin;
   }
@@ -225,7 +324,26 @@ __global__ void __launch_bounds__(256) k_plan(ModelDims md, StepDev s, int B) {
 }
 
 void launch_router(const ModelDims& md, const StepDev& s, int B, const void* emb, const void* router_w,
-                   const float* router_b, const PageUpdate* upd, const int* n_upd, cudaStream_t st) {
+                   const float* router_b, const PageUpdate* upd, const int* n_upd, cudaStream_t st,
+                   const void* router_w1, const float* router_b1) {
+  if (md.router_hidden > 0) {
+    const size_t smem = (size_t)(md.d + md.router_hidden) * 4;
+    static bool attr[2] = {false, false};
+    if (!attr[md.dtype]) {
+      if (md.dtype == 1)
+        cudaFuncSetAttribute(k_router_mlp<bf16>, cudaFuncAttributeMaxDynamicSharedMemorySize, 65536);
+      else
+        cudaFuncSetAttribute(k_router_mlp<float>, cudaFuncAttributeMaxDynamicSharedMemorySize, 65536);
+      attr[md.dtype] = true;
+    }
+    if (md.dtype == 1)
+      launch_k(k_router_mlp<bf16>, B, 256, smem, st, md, s, B, (const bf16*)emb, (const bf16*)router_w1, router_b1,
+               (const bf16*)router_w, router_b, upd, n_upd);
+    else
+      launch_k(k_router_mlp<float>, B, 256, smem, st, md, s, B, (const float*)emb, (const float*)router_w1,
+               router_b1, (const float*)router_w, router_b, upd, n_upd);
+    return;
+  }
   const int grid = (B + 7) / 8;
   if (md.dtype == 1)
     launch_k(k_router<bf16>, grid, 256, 0, st, md, s, B, (const bf16*)emb, (const bf16*)router_w, router_b, upd,

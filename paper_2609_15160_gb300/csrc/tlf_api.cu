@@ -58,6 +58,8 @@ struct tlf_ctx {
   // weights
   void* d_emb = nullptr;
   void* d_router_w = nullptr;
+  void* d_router_w1 = nullptr;   // MLP router hidden layer [H_r][d]
+  float* d_router_b1 = nullptr;
   float* d_router_b = nullptr;
   float* d_attn_norm = nullptr;
   float* d_mlp_norm = nullptr;
@@ -230,6 +232,9 @@ extern "C" int tlf_validate_config(const tlf_config* c, char* msg, size_t msg_le
   if (c->ablation == TLF_ABLATION_DENSE_CACHE && c->dtype != TLF_DTYPE_BF16)
     return bad("the dense-cache ablation needs a bf16 model");
   if (c->conditioning != 0 && c->conditioning != 1) return bad("conditioning must be 0 or 1");
+  if (c->router_hidden < 0 || c->router_hidden > 8192 || c->router_hidden % 8)
+    return bad("router_hidden must be 0 or a multiple of 8 up to 8192");
+  if (c->reserved != 0) return bad("reserved must be 0");
   if (msg && msg_len) snprintf(msg, msg_len, "ok");
   return TLF_OK;
 }
@@ -337,6 +342,7 @@ static int create_impl(tlf_ctx* ctx, const tlf_weights* w) {
   md.dtype = c.dtype;
   md.max_pos = c.max_seq_len;
   md.ablation = c.ablation;
+  md.router_hidden = c.router_hidden;
   ctx->eb = c.dtype == TLF_DTYPE_BF16 ? 2 : 4;
   md.page_elems = (long long)md.J * 2 * md.Hkv * md.page_size * md.hd;
   ctx->n_pages = c.kv_pool_pages > 0 ? c.kv_pool_pages : (int64_t)c.max_seqs * c.max_loops * md.max_pages;
@@ -373,7 +379,13 @@ static int create_impl(tlf_ctx* ctx, const tlf_weights* w) {
   const size_t eb = ctx->eb;
   const int d = md.d, J = md.J, ff = md.ff, V = md.V, M = md.M, B = md.max_batch;
   int rc;
-  if ((rc = upload(ctx, &ctx->d_router_w, w->router_w, (size_t)M * d * eb, "router_w"))) return rc;
+  const int Hr = c.router_hidden;
+  if ((rc = upload(ctx, &ctx->d_router_w, w->router_w, (size_t)M * (Hr > 0 ? Hr : d) * eb, "router_w"))) return rc;
+  if (Hr > 0) {
+    if (!w->router_w1 || !w->router_b1) return fail(ctx, TLF_ERR_BAD_WEIGHTS, "MLP router weights are NULL");
+    if ((rc = upload(ctx, &ctx->d_router_w1, w->router_w1, (size_t)Hr * d * eb, "router_w1"))) return rc;
+    if ((rc = upload(ctx, (void**)&ctx->d_router_b1, w->router_b1, (size_t)Hr * 4, "router_b1"))) return rc;
+  }
   if ((rc = upload(ctx, (void**)&ctx->d_router_b, w->router_b, (size_t)M * 4, "router_b"))) return rc;
   if ((rc = upload(ctx, (void**)&ctx->d_attn_norm, w->attn_norm, (size_t)J * d * 4, "attn_norm"))) return rc;
   if ((rc = upload(ctx, (void**)&ctx->d_mlp_norm, w->mlp_norm, (size_t)J * d * 4, "mlp_norm"))) return rc;
@@ -540,7 +552,7 @@ extern "C" void tlf_destroy(tlf_ctx* ctx) {
   if (!ctx->host_only) {
     cudaDeviceSynchronize();
     auto f = [](void* p) { if (p) cudaFree(p); };
-    f(ctx->d_emb); f(ctx->d_router_w); f(ctx->d_router_b); f(ctx->d_attn_norm); f(ctx->d_mlp_norm);
+    f(ctx->d_emb); f(ctx->d_router_w); f(ctx->d_router_w1); f(ctx->d_router_b1); f(ctx->d_router_b); f(ctx->d_attn_norm); f(ctx->d_mlp_norm);
     f(ctx->d_final_norm); f(ctx->d_inv_freq); f(ctx->d_rope); f(ctx->d_rowinfo); f(ctx->d_act); f(ctx->d_cond);
     for (auto* v : {&ctx->wqkv, &ctx->wo, &ctx->wgu, &ctx->wd})
       for (auto& m : *v) f(m.ptr);
@@ -730,7 +742,8 @@ static int enqueue_step(tlf_ctx* ctx, int B, bool need_logits, bool prof, cudaSt
     if (cls >= 0) ctx->ev_class.push_back(cls);
   };
   mark(-1);
-  launch_router(md, s, B, ctx->d_emb, ctx->d_router_w, ctx->d_router_b, d_upd, ctx->d_upload, st);
+  launch_router(md, s, B, ctx->d_emb, ctx->d_router_w, ctx->d_router_b, d_upd, ctx->d_upload, st, ctx->d_router_w1,
+                ctx->d_router_b1);
   mark(0);
   launch_plan(md, s, B, st);
   mark(1);
@@ -1116,7 +1129,8 @@ static int prefill_batched(tlf_ctx* ctx, int n_seqs, const int* slot_of, const i
     sr.page_table = ctx->d_page_table;
     sr.err = ctx->d_err;
     launch_router(md, sr, T, ctx->d_emb, ctx->d_router_w, ctx->d_router_b,
-                  reinterpret_cast<const PageUpdate*>(ctx->d_pf_in + 1 + 4 * C + 2 * Smax), ctx->d_pf_in, st);
+                  reinterpret_cast<const PageUpdate*>(ctx->d_pf_in + 1 + 4 * C + 2 * Smax), ctx->d_pf_in, st,
+                  ctx->d_router_w1, ctx->d_router_b1);
     PrefillDev P{};
     P.T = T;
     P.S = S;

@@ -335,6 +335,7 @@ struct ModelDims {
   int dtype;             // 0 f32, 1 bf16
   int max_pos;           // positions 0..max_pos-1 have a row in the rotary table
   int ablation;          // tlf_ablation
+  int router_hidden;     // > 0: two-layer MLP router with this hidden width
 };
 
 // Time/step conditioning (Sec. 3.1, App. A) inside the step. The modulation of
@@ -397,7 +398,8 @@ struct PageUpdate {
 };
 
 void launch_router(const ModelDims& md, const StepDev& s, int B, const void* emb, const void* router_w,
-                   const float* router_b, const PageUpdate* upd, const int* n_upd, cudaStream_t st);
+                   const float* router_b, const PageUpdate* upd, const int* n_upd, cudaStream_t st,
+                   const void* router_w1 = nullptr, const float* router_b1 = nullptr);
 void launch_plan(const ModelDims& md, const StepDev& s, int B, cudaStream_t st);
 
 void launch_norm_rows(int dtype, const float* H, int ldh, const int* idx, const int* n_dev, int n_host,

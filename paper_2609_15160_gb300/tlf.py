@@ -34,7 +34,8 @@ class TlfConfig(C.Structure):
         ("rope_base", C.c_float), ("norm_eps", C.c_float), ("dtype", C.c_int32), ("exit_rule", C.c_int32),
         ("threshold", C.c_float), ("max_seqs", C.c_int32), ("max_batch", C.c_int32), ("max_seq_len", C.c_int32),
         ("page_size", C.c_int32), ("gemm_impl", C.c_int32), ("host_only", C.c_int32), ("prefill_chunk", C.c_int32),
-        ("kv_pool_pages", C.c_int64), ("ablation", C.c_int32), ("conditioning", C.c_int32)]
+        ("kv_pool_pages", C.c_int64), ("ablation", C.c_int32), ("conditioning", C.c_int32),
+        ("router_hidden", C.c_int32), ("reserved", C.c_int32)]
 
 
 COND_WEIGHTS = ("cond_t_w1", "cond_t_b1", "cond_t_w2", "cond_t_b2", "cond_dt_w1", "cond_dt_b1", "cond_dt_w2",
@@ -43,7 +44,8 @@ COND_WEIGHTS = ("cond_t_w1", "cond_t_b1", "cond_t_w2", "cond_t_b2", "cond_dt_w1"
 
 class TlfWeights(C.Structure):
     _fields_ = [(n, C.c_void_p) for n in ("embedding", "router_w", "router_b", "wq", "wk", "wv", "wo", "w_gate",
-                                          "w_up", "w_down", "attn_norm", "mlp_norm", "final_norm") + COND_WEIGHTS]
+                                          "w_up", "w_down", "attn_norm", "mlp_norm", "final_norm") + COND_WEIGHTS
+                + ("router_w1", "router_b1")]
 
 
 class TlfAttnArgs(C.Structure):
@@ -151,7 +153,8 @@ def make_config(m, max_seqs: int, max_batch: int, max_seq_len: int, page_size: i
                      threshold=m.threshold, max_seqs=max_seqs, max_batch=max_batch, max_seq_len=max_seq_len,
                      page_size=page_size, gemm_impl=GEMM[gemm_impl], host_only=int(host_only), prefill_chunk=prefill_chunk,
                      kv_pool_pages=kv_pool_pages, ablation=ABLATION[ablation],
-                     conditioning=int(getattr(m, "conditioning", False)))
+                     conditioning=int(getattr(m, "conditioning", False)),
+                     router_hidden=int(getattr(m, "router_hidden", 0)))
 
 
 def tlf_validate_config(cfg: TlfConfig):
@@ -182,6 +185,9 @@ def tlf_create(cfg: TlfConfig, weights: Optional[Dict[str, np.ndarray]], dtype: 
         if cfg.conditioning:
             for name in COND_WEIGHTS:
                 keep[name] = np.ascontiguousarray(weights[name], dtype=np.float32)
+        if cfg.router_hidden:
+            keep["router_w1"] = _matrix(weights["router_w1"], dtype)
+            keep["router_b1"] = np.ascontiguousarray(weights["router_b1"], dtype=np.float32)
         for name, arr in keep.items():
             setattr(w, name, arr.ctypes.data)
     h = _P()

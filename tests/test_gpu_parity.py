@@ -2,6 +2,8 @@
 
 Every call goes through the C ABI (libtlf.so) via the ctypes binding.
 """
+import dataclasses
+
 import numpy as np
 import pytest
 
@@ -417,3 +419,31 @@ def test_conditioning_small_models(tlf, dtype, gemm_impl):
 
 def test_conditioning_with_no_gather(tlf):
     _prefill_decode_compare(tlf, _small(conditioning=True), [65, 3, 64], steps=3, ablation="no_gather")
+
+
+# ----------------------------------------------------------------------------
+# the two-layer MLP router (Sec. 3.2) and the survival rule at several thresholds (Eq. 4)
+# ----------------------------------------------------------------------------
+
+@pytest.mark.parametrize("dtype,gemm_impl,rule", [("bf16", "auto", "argmax"), ("bf16", "simt", "survival"),
+                                                  ("f32", "auto", "argmax")])
+def test_mlp_router_small_models(tlf, dtype, gemm_impl, rule):
+    m = _small(dtype, router_hidden=64, exit_rule=rule)
+    _prefill_decode_compare(tlf, m, [70, 1, 130], steps=4, gemm_impl=gemm_impl)
+
+
+def test_mlp_router_c3_shapes(tlf):
+    """C3 model with a 256-wide MLP router: every loop count and active set, sampled logits and caches."""
+    wl = synth.get_config("c3")
+    wl = dataclasses.replace(wl, model=dataclasses.replace(wl.model, router_hidden=256))
+    lengths = np.full(wl.batch, wl.prompt_len[0])
+    worst, forced = _snapshot_run(tlf, wl, lengths, steps=3, sampled=[0, 21])
+    print(f"c3 mlp router worst {worst:.2e} forced {forced}")
+
+
+@pytest.mark.parametrize("threshold", [0.2, 0.8])
+def test_survival_thresholds_c2(tlf, threshold):
+    wl = synth.get_config("c2").with_batch(4)
+    wl = dataclasses.replace(wl, model=dataclasses.replace(wl.model, exit_rule="survival", threshold=threshold))
+    worst, forced = _greedy_run(tlf, wl, steps=8)
+    print(f"c2 survival {threshold} worst {worst:.2e} forced {forced}")

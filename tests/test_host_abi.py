@@ -49,7 +49,7 @@ def _cfg(**kw):
 @pytest.mark.parametrize("field,value", [
     ("d_model", 100), ("n_kv_heads", 3), ("head_dim", 48), ("max_loops", 0), ("max_loops", 17),
     ("max_batch", 0), ("max_batch", 300), ("page_size", 32), ("dtype", 7), ("ffn_hidden", 1000),
-    ("exit_rule", 5), ("norm_eps", 0.0), ("max_seqs", 2), ("ablation", 9), ("conditioning", 2),
+    ("exit_rule", 5), ("norm_eps", 0.0), ("max_seqs", 2), ("ablation", 9), ("conditioning", 2), ("router_hidden", 12), ("router_hidden", 9000), ("reserved", 1),
 ])
 def test_validate_config_rejects(lib, field, value):
     rc, msg = tlf.tlf_validate_config(_cfg(**{field: value}))
@@ -59,7 +59,7 @@ def test_validate_config_rejects(lib, field, value):
 def test_config_struct_matches_the_header(lib):
     """The ctypes mirror of tlf_config has the C layout: int64 pool size at offset 80, then the ablation."""
     assert tlf.TlfConfig.kv_pool_pages.offset == 80 and tlf.TlfConfig.ablation.offset == 88
-    assert C.sizeof(tlf.TlfConfig) == 96
+    assert tlf.TlfConfig.router_hidden.offset == 96 and C.sizeof(tlf.TlfConfig) == 104
     for name in ("none", "no_gather"):
         rc, msg = tlf.tlf_validate_config(_cfg(ablation=tlf.ABLATION[name]))
         assert rc == 0, msg
