@@ -70,7 +70,7 @@ __global__ void __launch_bounds__(1024) k_pf_plan(ModelDims md, PrefillDev p) {
     const int v = tid < S ? cnt_s[tid] : 0;
     int n_r;
     const int first = pf_block_scan(v, &n_r, warp_tot);
-    const int qb = (v + PF_QB - 1) / PF_QB;
+    const int qb = (v + p.qblock - 1) / p.qblock;
     int tiles;
     const int tb = pf_block_scan(qb, &tiles, warp_tot);
     if (tid < S) {
@@ -243,6 +243,270 @@ __global__ void __launch_bounds__(32 * PF_WARPS) k_pf_attn(ModelDims md, Prefill
   }
 }
 
+// ----------------------------------------------------------------------------
+// Tensor-core causal attention of a chunk (bf16 models, head_dim 64 or 128)
+// ----------------------------------------------------------------------------
+// One CTA of 128 threads per (sequence, block of QT = 128/G queries, kv head): the 128 MMA rows
+// are the G query heads of QT queries (row = query * G + head). For every page of 64 cache slots:
+//   S = Q K^T   tcgen05.mma M=128, N=64, K=hd into TMEM; q enters as two bf16 terms (q = hi + lo),
+//               so the scores keep q's float32 precision;
+//   softmax     thread t owns row t: it reads the row of S (tcgen05.ld), masks causally by cache
+//               slot, and keeps an online softmax in float32 (base 2); P goes to shared memory in
+//               bf16, and the row sum adds the same rounded values;
+//   O += P V    tcgen05.mma M=128, N=hd, K=64 accumulating in TMEM.
+// The running maximum is refreshed lazily: O (TMEM load, scale, store) and the row sum are
+// rescaled only when a row's maximum grows by more than 8 (a factor of 256), so exponentials stay
+// below 256 and rescaling is rare. The K and V segments of each page arrive by 1-D bulk copies in
+// a two-deep staging ring; threads rewrite them into the swizzled K-major operand tiles (V
+// transposed so that keys run along K), with zeros past the last valid slot.
+constexpr int PFT_THREADS = 128;
+
+template <int HD>
+struct PfTcShape {
+  static constexpr int A_BYTES = 128 * HD * 2;   // one of the hi / lo Q tiles [128][HD]
+  static constexpr int BK_BYTES = 64 * HD * 2;   // K tile [64 keys][HD]
+  static constexpr int BV_BYTES = HD * 64 * 2;   // V^T tile [HD][64 keys]
+  static constexpr int P_BYTES = 128 * 64 * 2;   // P tile [128][64 keys]
+  static constexpr int SEG = 64 * HD * 2;        // raw K (or V) segment of a page
+  static constexpr int RAW_BYTES = 2 * SEG;
+  static constexpr int OFF_AHI = 0;
+  static constexpr int OFF_ALO = OFF_AHI + A_BYTES;
+  static constexpr int OFF_BK = OFF_ALO + A_BYTES;
+  static constexpr int OFF_BV = OFF_BK + BK_BYTES;
+  static constexpr int OFF_P = OFF_BV + BV_BYTES;
+  static constexpr int OFF_RAW = OFF_P + P_BYTES;
+  static constexpr int OFF_BAR = OFF_RAW + 2 * RAW_BYTES;
+  static constexpr int BYTES = OFF_BAR + 64 + 1024;   // barriers, TMEM slot, alignment slack
+  static constexpr uint32_t TMEM_COLS = 256;          // S in columns 0..63, O in 64..64+HD
+  static constexpr int ACOL = 128 * 128;              // bytes of one 128-byte atom column of a Q tile
+  static constexpr int BCOL = 64 * 128;               // ... of the K tile
+};
+
+__device__ __forceinline__ uint32_t pack_bf16(float a, float b) {
+  return (uint32_t)__bfloat16_as_ushort(__float2bfloat16_rn(a)) |
+         ((uint32_t)__bfloat16_as_ushort(__float2bfloat16_rn(b)) << 16);
+}
+
+template <int HD, int G>
+__global__ void __launch_bounds__(PFT_THREADS) k_pf_attn_tc(ModelDims md, PrefillDev p, StepDev s, int r, int j,
+                                                             const float* __restrict__ Q, bf16* __restrict__ O) {
+  using Sh = PfTcShape<HD>;
+  constexpr int QT = 128 / G;
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* sm = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+  uint64_t* bars = reinterpret_cast<uint64_t*>(sm + Sh::OFF_BAR);  // staging 0, staging 1, S done, O done
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 4);
+
+  pdl_wait();
+  pdl_trigger();
+  const int S = p.S;
+  const int* tbase = p.tile_base + r * (p.Smax + 1);
+  const int tile = blockIdx.x, kvh = blockIdx.y;
+  if (tile >= tbase[S]) return;
+  int lo = 0, hi = S;  // sequence: largest sq with tbase[sq] <= tile
+  while (hi - lo > 1) {
+    const int mid = (lo + hi) >> 1;
+    if (tbase[mid] <= tile) lo = mid; else hi = mid;
+  }
+  const int sq = lo, qb = tile - tbase[sq];
+  const int cnt = p.cnt[r * p.Smax + sq], first = p.first[r * p.Smax + sq], s0 = p.s0[r * p.Smax + sq];
+  const int slot = p.seq_slot[sq];
+  const int q0 = qb * QT, nq = min(QT, cnt - q0);
+  const int last = s0 + q0 + nq - 1;  // cache slot of the block's last query
+  const int npages = last / 64 + 1;
+  const int tid = threadIdx.x, warp = tid >> 5;
+  const int* ptab = s.page_table + ((size_t)slot * md.M + r) * md.max_pages;
+  const uint32_t stg0 = smem_u32(&bars[0]), stg1 = smem_u32(&bars[1]);
+  const uint32_t bar_s = smem_u32(&bars[2]), bar_o = smem_u32(&bars[3]);
+
+  if (tid == 0) {
+    for (int i = 0; i < 4; ++i) mbar_init(smem_u32(&bars[i]), 1);
+    fence_barrier_init();
+  }
+  if (warp == 0) {
+    tmem_alloc(smem_u32(tmem_slot), Sh::TMEM_COLS);
+    tmem_relinquish();
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = *tmem_slot;
+  const uint32_t t_row = tmem + ((uint32_t)(warp * 32) << 16);  // this warp's 32 TMEM lanes
+
+  auto stage_page = [&](int pg) {  // thread 0: K and V segments of page pg into staging buffer pg & 1
+    const uint32_t bar = (pg & 1) ? stg1 : stg0;
+    const int page = ptab[pg];
+    if (page < 0 || page >= md.n_pages) {
+      atomicOr(s.err, DEVERR_INDEX);
+      mbar_arrive(bar);  // complete the phase without data
+      return;
+    }
+    const bf16* kseg = reinterpret_cast<const bf16*>(s.pool) + (size_t)page * md.page_elems +
+                       ((size_t)(j * 2 + 0) * md.Hkv + kvh) * 64 * HD;
+    const bf16* vseg = kseg + (size_t)md.Hkv * 64 * HD;
+    uint8_t* dst = sm + Sh::OFF_RAW + (pg & 1) * Sh::RAW_BYTES;
+    mbar_arrive_expect_tx(bar, Sh::RAW_BYTES);
+    bulk_g2s(smem_u32(dst), kseg, Sh::SEG, bar);
+    bulk_g2s(smem_u32(dst + Sh::SEG), vseg, Sh::SEG, bar);
+  };
+  if (tid == 0) {
+    stage_page(0);
+    if (npages > 1) stage_page(1);
+  }
+
+  // Q tile rows: thread t writes row t as hi and lo bf16 parts (zeros past the block's queries)
+  const int qi = tid / G, g = tid % G;
+  const bool row_ok = qi < nq;
+  {
+    const float4* qrow = reinterpret_cast<const float4*>(Q + ((size_t)(first + q0 + qi) * md.Hq + kvh * G + g) * HD);
+#pragma unroll 4
+    for (int c = 0; c < HD / 8; ++c) {
+      float x[8];
+      if (row_ok) {
+        const float4 a = qrow[2 * c], b = qrow[2 * c + 1];
+        x[0] = a.x; x[1] = a.y; x[2] = a.z; x[3] = a.w; x[4] = b.x; x[5] = b.y; x[6] = b.z; x[7] = b.w;
+      } else {
+#pragma unroll
+        for (int u = 0; u < 8; ++u) x[u] = 0.f;
+      }
+      uint32_t h[4], l[4];
+#pragma unroll
+      for (int u = 0; u < 4; ++u) {
+        const float a0 = __bfloat162float(__float2bfloat16_rn(x[2 * u]));
+        const float a1 = __bfloat162float(__float2bfloat16_rn(x[2 * u + 1]));
+        h[u] = pack_bf16(a0, a1);
+        l[u] = pack_bf16(x[2 * u] - a0, x[2 * u + 1] - a1);
+      }
+      const uint32_t off = (c / 8) * Sh::ACOL + sw128_off(tid, c % 8);
+      *reinterpret_cast<uint4*>(sm + Sh::OFF_AHI + off) = make_uint4(h[0], h[1], h[2], h[3]);
+      *reinterpret_cast<uint4*>(sm + Sh::OFF_ALO + off) = make_uint4(l[0], l[1], l[2], l[3]);
+    }
+  }
+
+  const int qslot = s0 + q0 + qi;  // cache slot of this row's query
+  const float scale = 1.4426950408889634f * rsqrtf((float)HD);
+  constexpr uint32_t IDS = idesc_bf16_f32(128, 64), IDO = idesc_bf16_f32(128, HD);
+  float m_run = -INFINITY, l_run = 0.f;
+
+  for (int pg = 0; pg < npages; ++pg) {
+    if (pg > 0) mbar_wait(bar_o, (pg - 1) & 1, s.err);  // previous P V done: K, V^T and P tiles free
+    mbar_wait((pg & 1) ? stg1 : stg0, (pg >> 1) & 1, s.err);
+    const uint8_t* raw = sm + Sh::OFF_RAW + (pg & 1) * Sh::RAW_BYTES;
+    const int valid = min(64, last + 1 - pg * 64);
+    for (int e = tid; e < 64 * (HD / 8); e += PFT_THREADS) {  // K tile: row = key
+      const int key = e / (HD / 8), c = e % (HD / 8);
+      const uint4 v = key < valid ? *reinterpret_cast<const uint4*>(raw + key * HD * 2 + c * 16) : make_uint4(0, 0, 0, 0);
+      *reinterpret_cast<uint4*>(sm + Sh::OFF_BK + (c / 8) * Sh::BCOL + sw128_off(key, c % 8)) = v;
+    }
+    const unsigned short* rv = reinterpret_cast<const unsigned short*>(raw + Sh::SEG);
+    for (int e = tid; e < HD * 8; e += PFT_THREADS) {  // V^T tile: row = hd index n, chunk c = keys 8c..8c+7
+      const int n = e % HD, c = e / HD;
+      uint32_t w[4];
+#pragma unroll
+      for (int u = 0; u < 4; ++u) {
+        const int k0 = 8 * c + 2 * u;
+        const uint32_t b0 = k0 < valid ? rv[k0 * HD + n] : 0u;
+        const uint32_t b1 = k0 + 1 < valid ? rv[(k0 + 1) * HD + n] : 0u;
+        w[u] = b0 | (b1 << 16);
+      }
+      *reinterpret_cast<uint4*>(sm + Sh::OFF_BV + sw128_off(n, c)) = make_uint4(w[0], w[1], w[2], w[3]);
+    }
+    fence_proxy_async_smem();
+    __syncthreads();
+    if (tid == 0) {
+      if (pg + 2 < npages) stage_page(pg + 2);  // this staging buffer has been read
+      tc_fence_after();
+#pragma unroll
+      for (int kc = 0; kc < HD / 64; ++kc)
+#pragma unroll
+        for (int k = 0; k < 4; ++k) {  // K = 16 per MMA: +32 bytes (encoded +2) inside the atom column
+          const uint64_t db = smem_desc_sw128(smem_u32(sm + Sh::OFF_BK + kc * Sh::BCOL)) + 2 * k;
+          tc_mma_f16(tmem, smem_desc_sw128(smem_u32(sm + Sh::OFF_AHI + kc * Sh::ACOL)) + 2 * k, db, IDS,
+                     (kc | k) ? 1u : 0u);
+          tc_mma_f16(tmem, smem_desc_sw128(smem_u32(sm + Sh::OFF_ALO + kc * Sh::ACOL)) + 2 * k, db, IDS, 1u);
+        }
+      tc_commit(bar_s);
+    }
+    __syncwarp();
+    mbar_wait(bar_s, pg & 1, s.err);
+    tc_fence_after();
+
+    float sc[64];
+#pragma unroll
+    for (int c0 = 0; c0 < 64; c0 += 16) tmem_ld_16(t_row + c0, sc + c0);
+    float pm = -INFINITY;
+#pragma unroll
+    for (int c = 0; c < 64; ++c) {
+      const bool use = row_ok && c < valid && pg * 64 + c <= qslot;  // causal by cache slot
+      sc[c] = use ? sc[c] * scale : -INFINITY;
+      pm = fmaxf(pm, sc[c]);
+    }
+    // lazy maximum: rescale only when it grows by more than 8 (warp-uniform TMEM access)
+    const bool grow = pm > m_run + 8.f;
+    const float cr = grow ? exp2f(m_run - pm) : 1.f;  // 0 when m_run was -inf
+    if (__any_sync(0xffffffffu, grow) && pg > 0) {
+#pragma unroll
+      for (int c0 = 0; c0 < HD; c0 += 16) {
+        float o[16];
+        tmem_ld_16(t_row + 64 + c0, o);
+#pragma unroll
+        for (int i = 0; i < 16; ++i) o[i] *= cr;
+        tmem_st_16(t_row + 64 + c0, o);
+      }
+    }
+    if (grow) {
+      l_run *= cr;
+      m_run = pm;
+    }
+    uint32_t pk[32];
+    float psum = 0.f;
+#pragma unroll
+    for (int c = 0; c < 64; c += 2) {
+      const float p0 = sc[c] == -INFINITY ? 0.f : exp2f(sc[c] - m_run);
+      const float p1 = sc[c + 1] == -INFINITY ? 0.f : exp2f(sc[c + 1] - m_run);
+      pk[c / 2] = pack_bf16(p0, p1);
+      psum += __bfloat162float(__ushort_as_bfloat16((unsigned short)(pk[c / 2] & 0xFFFFu))) +
+              __bfloat162float(__ushort_as_bfloat16((unsigned short)(pk[c / 2] >> 16)));
+    }
+    l_run += psum;
+#pragma unroll
+    for (int q = 0; q < 8; ++q)
+      *reinterpret_cast<uint4*>(sm + Sh::OFF_P + sw128_off(tid, q)) =
+          make_uint4(pk[4 * q], pk[4 * q + 1], pk[4 * q + 2], pk[4 * q + 3]);
+    fence_proxy_async_smem();
+    tc_fence_before();
+    __syncthreads();
+    if (tid == 0) {
+      tc_fence_after();
+#pragma unroll
+      for (int k = 0; k < 4; ++k)
+        tc_mma_f16(tmem + 64, smem_desc_sw128(smem_u32(sm + Sh::OFF_P)) + 2 * k,
+                   smem_desc_sw128(smem_u32(sm + Sh::OFF_BV)) + 2 * k, IDO, (pg > 0 || k > 0) ? 1u : 0u);
+      tc_commit(bar_o);
+    }
+    __syncwarp();
+  }
+  mbar_wait(bar_o, (npages - 1) & 1, s.err);
+  tc_fence_after();
+  const float inv_l = l_run > 0.f ? 1.f / l_run : 0.f;
+  bf16* orow = O + (size_t)(first + q0 + qi) * md.q_dim + (kvh * G + g) * HD;
+#pragma unroll
+  for (int c0 = 0; c0 < HD; c0 += 16) {
+    float o[16];
+    tmem_ld_16(t_row + 64 + c0, o);
+    if (row_ok) {
+      uint32_t w[8];
+#pragma unroll
+      for (int i = 0; i < 8; ++i) w[i] = pack_bf16(o[2 * i] * inv_l, o[2 * i + 1] * inv_l);
+      *reinterpret_cast<uint4*>(orow + c0) = make_uint4(w[0], w[1], w[2], w[3]);
+      *reinterpret_cast<uint4*>(orow + c0 + 8) = make_uint4(w[4], w[5], w[6], w[7]);
+    }
+  }
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 0) tmem_dealloc(tmem, Sh::TMEM_COLS);
+}
+
 __global__ void k_pf_len(ModelDims md, PrefillDev p) {
   pdl_wait();
   pdl_trigger();
@@ -268,15 +532,33 @@ void launch_pf_plan(const ModelDims& md, const PrefillDev& p, cudaStream_t st) {
   launch_k(k_pf_plan, 1, 1024, 0, st, md, p);
 }
 
+template <int HD, int G>
+static void pf_attn_tc_launch(const ModelDims& md, const PrefillDev& p, const StepDev& s, int r, int j,
+                              const float* Q, void* O, int tiles_bound, cudaStream_t st) {
+  static bool attr = false;
+  constexpr int smem = PfTcShape<HD>::BYTES;
+  if (!attr) {
+    cudaFuncSetAttribute(k_pf_attn_tc<HD, G>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+    attr = true;
+  }
+  launch_k(k_pf_attn_tc<HD, G>, dim3(tiles_bound, md.Hkv), PFT_THREADS, smem, st, md, p, s, r, j, Q, (bf16*)O);
+}
+
+// Tensor-core kernel for head_dim 64 and 128 (128-byte rows for the swizzled operand tiles); the
+// CUDA-core kernel for head_dim 32.
+static bool pf_attn_uses_tc(const ModelDims& md) { return md.hd == 64 || md.hd == 128; }
+
+int pf_attn_qblock(const ModelDims& md) { return pf_attn_uses_tc(md) ? 128 / (md.Hq / md.Hkv) : PF_QB; }
+
 void launch_pf_attn(const ModelDims& md, const PrefillDev& p, const StepDev& s, int r, int j, const float* Q,
                     void* O, int tiles_bound, cudaStream_t st) {
   const int G = md.Hq / md.Hkv;
-  if (md.hd == 128 && G == 1) pf_attn_launch<bf16, 128, 1>(md, p, s, r, j, Q, O, tiles_bound, st);
-  else if (md.hd == 128 && G == 2) pf_attn_launch<bf16, 128, 2>(md, p, s, r, j, Q, O, tiles_bound, st);
-  else if (md.hd == 128 && G == 4) pf_attn_launch<bf16, 128, 4>(md, p, s, r, j, Q, O, tiles_bound, st);
-  else if (md.hd == 64 && G == 1) pf_attn_launch<bf16, 64, 1>(md, p, s, r, j, Q, O, tiles_bound, st);
-  else if (md.hd == 64 && G == 2) pf_attn_launch<bf16, 64, 2>(md, p, s, r, j, Q, O, tiles_bound, st);
-  else if (md.hd == 64 && G == 4) pf_attn_launch<bf16, 64, 4>(md, p, s, r, j, Q, O, tiles_bound, st);
+  if (md.hd == 128 && G == 1) pf_attn_tc_launch<128, 1>(md, p, s, r, j, Q, O, tiles_bound, st);
+  else if (md.hd == 128 && G == 2) pf_attn_tc_launch<128, 2>(md, p, s, r, j, Q, O, tiles_bound, st);
+  else if (md.hd == 128 && G == 4) pf_attn_tc_launch<128, 4>(md, p, s, r, j, Q, O, tiles_bound, st);
+  else if (md.hd == 64 && G == 1) pf_attn_tc_launch<64, 1>(md, p, s, r, j, Q, O, tiles_bound, st);
+  else if (md.hd == 64 && G == 2) pf_attn_tc_launch<64, 2>(md, p, s, r, j, Q, O, tiles_bound, st);
+  else if (md.hd == 64 && G == 4) pf_attn_tc_launch<64, 4>(md, p, s, r, j, Q, O, tiles_bound, st);
   else if (md.hd == 32 && G == 1) pf_attn_launch<bf16, 32, 1>(md, p, s, r, j, Q, O, tiles_bound, st);
   else pf_attn_launch<bf16, 32, 2>(md, p, s, r, j, Q, O, tiles_bound, st);
 }

@@ -1149,6 +1149,7 @@ static int prefill_batched(tlf_ctx* ctx, int n_seqs, const int* slot_of, const i
     P.cnt = ctx->d_pf_cnt;
     P.s0 = ctx->d_pf_s0;
     P.tile_base = ctx->d_pf_tile_base;
+    P.qblock = pf_attn_qblock(md);
     P.len = ctx->d_len;
     launch_pf_plan(md, P, st);
     StepDev sp{};
@@ -1176,7 +1177,7 @@ static int prefill_batched(tlf_ctx* ctx, int n_seqs, const int* slot_of, const i
         a.row_cslot = ctx->d_pf_row_cslot + (size_t)r * C;
         a.row_pos = ctx->d_pf_row_pos + (size_t)r * C;
         gemm_pf(ctx, ctx->wqkv[j], &ctx->pf_map_X, a, st);
-        launch_pf_attn(md, P, sp, r, j, ctx->d_pf_Q, ctx->d_pf_O, C / 32 + S + 1, st);
+        launch_pf_attn(md, P, sp, r, j, ctx->d_pf_Q, ctx->d_pf_O, C / P.qblock + S + 1, st);
         a = GemmArgs{};
         a.n_dev = n_dev;
         a.epi = EPI_CL_RESID;

@@ -221,6 +221,33 @@ __device__ __forceinline__ void tmem_ld_16(uint32_t taddr, float* v) {
   for (int i = 0; i < 16; ++i) v[i] = __uint_as_float(r[i]);
 }
 
+// 32 lanes x 32-bit, 16 consecutive columns per thread, register -> TMEM; waits for completion.
+__device__ __forceinline__ void tmem_st_16(uint32_t taddr, const float* v) {
+  asm volatile(
+      "tcgen05.st.sync.aligned.32x32b.x16.b32 [%0], "
+      "{%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,%16};" ::"r"(taddr),
+      "r"(__float_as_uint(v[0])), "r"(__float_as_uint(v[1])), "r"(__float_as_uint(v[2])), "r"(__float_as_uint(v[3])),
+      "r"(__float_as_uint(v[4])), "r"(__float_as_uint(v[5])), "r"(__float_as_uint(v[6])), "r"(__float_as_uint(v[7])),
+      "r"(__float_as_uint(v[8])), "r"(__float_as_uint(v[9])), "r"(__float_as_uint(v[10])), "r"(__float_as_uint(v[11])),
+      "r"(__float_as_uint(v[12])), "r"(__float_as_uint(v[13])), "r"(__float_as_uint(v[14])),
+      "r"(__float_as_uint(v[15]))
+      : "memory");
+  asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory");
+}
+
+// Makes this thread's ordinary shared-memory stores visible to the tensor cores
+// (the async proxy) once a barrier orders them before the MMA issue.
+__device__ __forceinline__ void fence_proxy_async_smem() {
+  asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+}
+
+// Byte offset of 16-byte chunk q of row `row` in a K-major tile with 128-byte
+// swizzling (rows of 128 B = 64 bf16, 8-row atoms; the tile base is 1024-byte
+// aligned), the layout TMA writes with CU_TENSOR_MAP_SWIZZLE_128B.
+__host__ __device__ constexpr uint32_t sw128_off(int row, int q) {
+  return (uint32_t)row * 128u + (uint32_t)((q ^ (row & 7)) << 4);
+}
+
 // Shared-memory matrix descriptor for a K-major operand tile written by TMA with
 // 128-byte swizzling: rows of 128 B, 8-row swizzle atoms 1024 B apart.
 __device__ __forceinline__ uint64_t smem_desc_sw128(uint32_t saddr) {
@@ -456,12 +483,15 @@ struct PrefillDev {
   int* cnt;            // [M][Smax] compact rows of each sequence
   int* s0;             // [M][Smax] loop-r cache length of each sequence before the chunk
   int* tile_base;      // [M][Smax + 1] attention query blocks, prefix over sequences
+  int qblock;          // queries per attention block (the attention kernel's tile)
   int* len;            // [max_seqs][M] cache lengths
 };
 void launch_pf_plan(const ModelDims& md, const PrefillDev& p, cudaStream_t st);
 void launch_pf_attn(const ModelDims& md, const PrefillDev& p, const StepDev& s, int r, int j, const float* Q,
                     void* O, int tiles_bound, cudaStream_t st);
 void launch_pf_len(const ModelDims& md, const PrefillDev& p, cudaStream_t st);
+// Queries per block of the prefill attention kernel that launch_pf_attn picks for this model.
+int pf_attn_qblock(const ModelDims& md);
 
 // Kernel-level attention operation (tlf_attn_decode): scratch layout and launch.
 struct AttnOpLayout {
