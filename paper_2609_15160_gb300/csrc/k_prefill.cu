@@ -246,20 +246,25 @@ __global__ void __launch_bounds__(32 * PF_WARPS) k_pf_attn(ModelDims md, Prefill
 // ----------------------------------------------------------------------------
 // Tensor-core causal attention of a chunk (bf16 models, head_dim 64 or 128)
 // ----------------------------------------------------------------------------
-// One CTA of 128 threads per (sequence, block of QT = 128/G queries, kv head): the 128 MMA rows
+// One CTA of 256 threads per (sequence, block of QT = 128/G queries, kv head): the 128 MMA rows
 // are the G query heads of QT queries (row = query * G + head). For every page of 64 cache slots:
 //   S = Q K^T   tcgen05.mma M=128, N=64, K=hd into TMEM; q enters as two bf16 terms (q = hi + lo),
 //               so the scores keep q's float32 precision;
-//   softmax     thread t owns row t: it reads the row of S (tcgen05.ld), masks causally by cache
-//               slot, and keeps an online softmax in float32 (base 2); P goes to shared memory in
-//               bf16, and the row sum adds the same rounded values;
+//   softmax     two threads share a row (warps w and w+4 reach the same TMEM lanes), each owning
+//               32 of its 64 columns: they read S (tcgen05.ld), mask causally by cache slot (only
+//               pages on the query's diagonal need the per-key test), exchange the row maximum
+//               through shared memory and keep an online softmax in float32 (base 2); P goes to
+//               shared memory in bf16;
 //   O += P V    tcgen05.mma M=128, N=hd, K=64 accumulating in TMEM.
+// The loop is software-pipelined: S has two TMEM buffers and the K / V^T operand tiles two
+// shared-memory buffers, so the S product of page p+1 runs on the tensor cores while the threads
+// do the softmax of page p, and the re-layout of page p+1 overlaps the P V product of page p.
 // The running maximum is refreshed lazily: O (TMEM load, scale, store) and the row sum are
 // rescaled only when a row's maximum grows by more than 8 (a factor of 256), so exponentials stay
 // below 256 and rescaling is rare. The K and V segments of each page arrive by 1-D bulk copies in
 // a two-deep staging ring; threads rewrite them into the swizzled K-major operand tiles (V
 // transposed so that keys run along K), with zeros past the last valid slot.
-constexpr int PFT_THREADS = 128;
+constexpr int PFT_THREADS = 256;
 
 template <int HD>
 struct PfTcShape {
@@ -271,16 +276,25 @@ struct PfTcShape {
   static constexpr int RAW_BYTES = 2 * SEG;
   static constexpr int OFF_AHI = 0;
   static constexpr int OFF_ALO = OFF_AHI + A_BYTES;
-  static constexpr int OFF_BK = OFF_ALO + A_BYTES;
-  static constexpr int OFF_BV = OFF_BK + BK_BYTES;
-  static constexpr int OFF_P = OFF_BV + BV_BYTES;
+  static constexpr int OFF_BK = OFF_ALO + A_BYTES;   // two K tiles
+  static constexpr int OFF_BV = OFF_BK + 2 * BK_BYTES;  // two V^T tiles
+  static constexpr int OFF_P = OFF_BV + 2 * BV_BYTES;
   static constexpr int OFF_RAW = OFF_P + P_BYTES;
   static constexpr int OFF_BAR = OFF_RAW + 2 * RAW_BYTES;
-  static constexpr int BYTES = OFF_BAR + 64 + 1024;   // barriers, TMEM slot, alignment slack
-  static constexpr uint32_t TMEM_COLS = 256;          // S in columns 0..63, O in 64..64+HD
+  static constexpr int OFF_XCH = OFF_BAR + 64;         // [2][128] floats: row maxima, then row sums
+  static constexpr int BYTES = OFF_XCH + 1024 + 1024;  // exchange, alignment slack
+  static constexpr uint32_t TMEM_COLS = 256;          // S buffers in columns 0..127, O in 128..128+HD
   static constexpr int ACOL = 128 * 128;              // bytes of one 128-byte atom column of a Q tile
-  static constexpr int BCOL = 64 * 128;               // ... of the K tile
+  static constexpr int BCOL = 64 * 128;               // ... of a K tile
 };
+
+// 2^x with the hardware approximation (relative error ~2^-22; the probabilities are then rounded
+// to bf16)
+__device__ __forceinline__ float ex2_approx(float x) {
+  float y;
+  asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
+  return y;
+}
 
 __device__ __forceinline__ uint32_t pack_bf16(float a, float b) {
   return (uint32_t)__bfloat16_as_ushort(__float2bfloat16_rn(a)) |
@@ -294,8 +308,9 @@ __global__ void __launch_bounds__(PFT_THREADS) k_pf_attn_tc(ModelDims md, Prefil
   constexpr int QT = 128 / G;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* sm = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
-  uint64_t* bars = reinterpret_cast<uint64_t*>(sm + Sh::OFF_BAR);  // staging 0, staging 1, S done, O done
-  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 4);
+  // staging 0, staging 1, S buffer 0 done, S buffer 1 done, P V done
+  uint64_t* bars = reinterpret_cast<uint64_t*>(sm + Sh::OFF_BAR);
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 5);
 
   pdl_wait();
   pdl_trigger();
@@ -314,13 +329,16 @@ __global__ void __launch_bounds__(PFT_THREADS) k_pf_attn_tc(ModelDims md, Prefil
   const int q0 = qb * QT, nq = min(QT, cnt - q0);
   const int last = s0 + q0 + nq - 1;  // cache slot of the block's last query
   const int npages = last / 64 + 1;
-  const int tid = threadIdx.x, warp = tid >> 5;
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  const int quad = warp & 3, half = warp >> 2;  // TMEM lane quadrant and column half of this warp
+  const int row = quad * 32 + lane;             // the MMA row (query * G + head) this thread serves
+  float* xch = reinterpret_cast<float*>(sm + Sh::OFF_XCH);
   const int* ptab = s.page_table + ((size_t)slot * md.M + r) * md.max_pages;
   const uint32_t stg0 = smem_u32(&bars[0]), stg1 = smem_u32(&bars[1]);
-  const uint32_t bar_s = smem_u32(&bars[2]), bar_o = smem_u32(&bars[3]);
+  const uint32_t bar_s0 = smem_u32(&bars[2]), bar_s1 = smem_u32(&bars[3]), bar_o = smem_u32(&bars[4]);
 
   if (tid == 0) {
-    for (int i = 0; i < 4; ++i) mbar_init(smem_u32(&bars[i]), 1);
+    for (int i = 0; i < 5; ++i) mbar_init(smem_u32(&bars[i]), 1);
     fence_barrier_init();
   }
   if (warp == 0) {
@@ -331,7 +349,8 @@ __global__ void __launch_bounds__(PFT_THREADS) k_pf_attn_tc(ModelDims md, Prefil
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem = *tmem_slot;
-  const uint32_t t_row = tmem + ((uint32_t)(warp * 32) << 16);  // this warp's 32 TMEM lanes
+  const uint32_t t_row = tmem + ((uint32_t)(quad * 32) << 16);  // this warp's 32 TMEM lanes
+  constexpr uint32_t OCOL = 128;                                 // first TMEM column of O
 
   auto stage_page = [&](int pg) {  // thread 0: K and V segments of page pg into staging buffer pg & 1
     const uint32_t bar = (pg & 1) ? stg1 : stg0;
@@ -349,151 +368,203 @@ __global__ void __launch_bounds__(PFT_THREADS) k_pf_attn_tc(ModelDims md, Prefil
     bulk_g2s(smem_u32(dst), kseg, Sh::SEG, bar);
     bulk_g2s(smem_u32(dst + Sh::SEG), vseg, Sh::SEG, bar);
   };
+  // K tile of page pg (from its staging buffer) into K buffer pg & 1; rows = keys
+  auto relayout_k = [&](int pg) {
+    mbar_wait((pg & 1) ? stg1 : stg0, (pg >> 1) & 1, s.err);
+    const uint8_t* raw = sm + Sh::OFF_RAW + (pg & 1) * Sh::RAW_BYTES;
+    uint8_t* bk = sm + Sh::OFF_BK + (pg & 1) * Sh::BK_BYTES;
+    const int valid = min(64, last + 1 - pg * 64);
+    for (int e = tid; e < 64 * (HD / 8); e += PFT_THREADS) {
+      const int key = e / (HD / 8), c = e % (HD / 8);
+      const uint4 v = key < valid ? *reinterpret_cast<const uint4*>(raw + key * HD * 2 + c * 16) : make_uint4(0, 0, 0, 0);
+      *reinterpret_cast<uint4*>(bk + (c / 8) * Sh::BCOL + sw128_off(key, c % 8)) = v;
+    }
+  };
+  // V^T tile of page pg into V buffer pg & 1: row = hd index n, chunk c = keys 8c..8c+7
+  auto relayout_v = [&](int pg) {
+    const uint8_t* raw = sm + Sh::OFF_RAW + (pg & 1) * Sh::RAW_BYTES;
+    uint8_t* bv = sm + Sh::OFF_BV + (pg & 1) * Sh::BV_BYTES;
+    const int valid = min(64, last + 1 - pg * 64);
+    const uint32_t* rv = reinterpret_cast<const uint32_t*>(raw + Sh::SEG);  // [64 keys][HD / 2] pairs
+    for (int e = tid; e < (HD / 2) * 8; e += PFT_THREADS) {
+      const int n2 = e % (HD / 2), c = e / (HD / 2);  // hd indices 2 n2, 2 n2 + 1; keys 8c..8c+7
+      uint32_t x[8];
+#pragma unroll
+      for (int u = 0; u < 8; ++u) x[u] = 8 * c + u < valid ? rv[(8 * c + u) * (HD / 2) + n2] : 0u;
+      uint32_t we[4], wo[4];
+#pragma unroll
+      for (int u = 0; u < 4; ++u) {
+        we[u] = __byte_perm(x[2 * u], x[2 * u + 1], 0x5410);  // low halves: hd index 2 n2
+        wo[u] = __byte_perm(x[2 * u], x[2 * u + 1], 0x7632);  // high halves: hd index 2 n2 + 1
+      }
+      *reinterpret_cast<uint4*>(bv + sw128_off(2 * n2, c)) = make_uint4(we[0], we[1], we[2], we[3]);
+      *reinterpret_cast<uint4*>(bv + sw128_off(2 * n2 + 1, c)) = make_uint4(wo[0], wo[1], wo[2], wo[3]);
+    }
+  };
+  constexpr uint32_t IDS = idesc_bf16_f32(128, 64), IDO = idesc_bf16_f32(128, HD);
+  auto issue_s = [&](int pg) {  // thread 0: S of page pg into TMEM columns 64 * (pg & 1)
+    tc_fence_after();
+    const uint32_t bk = smem_u32(sm + Sh::OFF_BK + (pg & 1) * Sh::BK_BYTES);
+#pragma unroll
+    for (int kc = 0; kc < HD / 64; ++kc)
+#pragma unroll
+      for (int k = 0; k < 4; ++k) {  // K = 16 per MMA: +32 bytes (encoded +2) inside the atom column
+        const uint64_t db = smem_desc_sw128(bk + kc * Sh::BCOL) + 2 * k;
+        const uint32_t d = tmem + 64u * (uint32_t)(pg & 1);
+        tc_mma_f16(d, smem_desc_sw128(smem_u32(sm + Sh::OFF_AHI + kc * Sh::ACOL)) + 2 * k, db, IDS, (kc | k) ? 1u : 0u);
+        tc_mma_f16(d, smem_desc_sw128(smem_u32(sm + Sh::OFF_ALO + kc * Sh::ACOL)) + 2 * k, db, IDS, 1u);
+      }
+    tc_commit((pg & 1) ? bar_s1 : bar_s0);
+  };
+
   if (tid == 0) {
     stage_page(0);
     if (npages > 1) stage_page(1);
   }
 
-  // Q tile rows: thread t writes row t as hi and lo bf16 parts (zeros past the block's queries)
-  const int qi = tid / G, g = tid % G;
-  const bool row_ok = qi < nq;
-  {
-    const float4* qrow = reinterpret_cast<const float4*>(Q + ((size_t)(first + q0 + qi) * md.Hq + kvh * G + g) * HD);
-#pragma unroll 4
-    for (int c = 0; c < HD / 8; ++c) {
-      float x[8];
-      if (row_ok) {
-        const float4 a = qrow[2 * c], b = qrow[2 * c + 1];
-        x[0] = a.x; x[1] = a.y; x[2] = a.z; x[3] = a.w; x[4] = b.x; x[5] = b.y; x[6] = b.z; x[7] = b.w;
-      } else {
+  // Q tile: row = query * G + head, as hi and lo bf16 parts (zeros past the block's queries)
+  for (int e = tid; e < 128 * (HD / 8); e += PFT_THREADS) {
+    const int qr = e / (HD / 8), c = e % (HD / 8);
+    const int qq = qr / G, gg = qr % G;
+    float x[8];
+    if (qq < nq) {
+      const float4* q4 = reinterpret_cast<const float4*>(Q + ((size_t)(first + q0 + qq) * md.Hq + kvh * G + gg) * HD);
+      const float4 a = q4[2 * c], b = q4[2 * c + 1];
+      x[0] = a.x; x[1] = a.y; x[2] = a.z; x[3] = a.w; x[4] = b.x; x[5] = b.y; x[6] = b.z; x[7] = b.w;
+    } else {
 #pragma unroll
-        for (int u = 0; u < 8; ++u) x[u] = 0.f;
-      }
-      uint32_t h[4], l[4];
-#pragma unroll
-      for (int u = 0; u < 4; ++u) {
-        const float a0 = __bfloat162float(__float2bfloat16_rn(x[2 * u]));
-        const float a1 = __bfloat162float(__float2bfloat16_rn(x[2 * u + 1]));
-        h[u] = pack_bf16(a0, a1);
-        l[u] = pack_bf16(x[2 * u] - a0, x[2 * u + 1] - a1);
-      }
-      const uint32_t off = (c / 8) * Sh::ACOL + sw128_off(tid, c % 8);
-      *reinterpret_cast<uint4*>(sm + Sh::OFF_AHI + off) = make_uint4(h[0], h[1], h[2], h[3]);
-      *reinterpret_cast<uint4*>(sm + Sh::OFF_ALO + off) = make_uint4(l[0], l[1], l[2], l[3]);
+      for (int u = 0; u < 8; ++u) x[u] = 0.f;
     }
+    uint32_t h[4], l[4];
+#pragma unroll
+    for (int u = 0; u < 4; ++u) {
+      const float a0 = __bfloat162float(__float2bfloat16_rn(x[2 * u]));
+      const float a1 = __bfloat162float(__float2bfloat16_rn(x[2 * u + 1]));
+      h[u] = pack_bf16(a0, a1);
+      l[u] = pack_bf16(x[2 * u] - a0, x[2 * u + 1] - a1);
+    }
+    const uint32_t off = (c / 8) * Sh::ACOL + sw128_off(qr, c % 8);
+    *reinterpret_cast<uint4*>(sm + Sh::OFF_AHI + off) = make_uint4(h[0], h[1], h[2], h[3]);
+    *reinterpret_cast<uint4*>(sm + Sh::OFF_ALO + off) = make_uint4(l[0], l[1], l[2], l[3]);
   }
+  const int qi = row / G, g = row % G;
+  const bool row_ok = qi < nq;
+  // prologue: page 0's operand tiles and its S product
+  relayout_k(0);
+  relayout_v(0);
+  fence_proxy_async_smem();
+  __syncthreads();
+  if (tid == 0) {
+    if (npages > 2) stage_page(2);  // staging buffer 0 has been read
+    issue_s(0);
+  }
+  __syncwarp();
 
   const int qslot = s0 + q0 + qi;  // cache slot of this row's query
   const float scale = 1.4426950408889634f * rsqrtf((float)HD);
-  constexpr uint32_t IDS = idesc_bf16_f32(128, 64), IDO = idesc_bf16_f32(128, HD);
   float m_run = -INFINITY, l_run = 0.f;
 
   for (int pg = 0; pg < npages; ++pg) {
-    if (pg > 0) mbar_wait(bar_o, (pg - 1) & 1, s.err);  // previous P V done: K, V^T and P tiles free
-    mbar_wait((pg & 1) ? stg1 : stg0, (pg >> 1) & 1, s.err);
-    const uint8_t* raw = sm + Sh::OFF_RAW + (pg & 1) * Sh::RAW_BYTES;
-    const int valid = min(64, last + 1 - pg * 64);
-    for (int e = tid; e < 64 * (HD / 8); e += PFT_THREADS) {  // K tile: row = key
-      const int key = e / (HD / 8), c = e % (HD / 8);
-      const uint4 v = key < valid ? *reinterpret_cast<const uint4*>(raw + key * HD * 2 + c * 16) : make_uint4(0, 0, 0, 0);
-      *reinterpret_cast<uint4*>(sm + Sh::OFF_BK + (c / 8) * Sh::BCOL + sw128_off(key, c % 8)) = v;
-    }
-    const unsigned short* rv = reinterpret_cast<const unsigned short*>(raw + Sh::SEG);
-    for (int e = tid; e < HD * 8; e += PFT_THREADS) {  // V^T tile: row = hd index n, chunk c = keys 8c..8c+7
-      const int n = e % HD, c = e / HD;
-      uint32_t w[4];
-#pragma unroll
-      for (int u = 0; u < 4; ++u) {
-        const int k0 = 8 * c + 2 * u;
-        const uint32_t b0 = k0 < valid ? rv[k0 * HD + n] : 0u;
-        const uint32_t b1 = k0 + 1 < valid ? rv[(k0 + 1) * HD + n] : 0u;
-        w[u] = b0 | (b1 << 16);
-      }
-      *reinterpret_cast<uint4*>(sm + Sh::OFF_BV + sw128_off(n, c)) = make_uint4(w[0], w[1], w[2], w[3]);
-    }
+    const bool more = pg + 1 < npages;
+    // operand tiles of page pg+1: its K buffer was last read by S of page pg-1 (complete), its V^T
+    // buffer by P V of page pg-1, which also frees P and lets O be rescaled
+    if (more) relayout_k(pg + 1);
+    if (pg > 0) mbar_wait(bar_o, (pg - 1) & 1, s.err);
+    if (more) relayout_v(pg + 1);
     fence_proxy_async_smem();
     __syncthreads();
-    if (tid == 0) {
-      if (pg + 2 < npages) stage_page(pg + 2);  // this staging buffer has been read
-      tc_fence_after();
-#pragma unroll
-      for (int kc = 0; kc < HD / 64; ++kc)
-#pragma unroll
-        for (int k = 0; k < 4; ++k) {  // K = 16 per MMA: +32 bytes (encoded +2) inside the atom column
-          const uint64_t db = smem_desc_sw128(smem_u32(sm + Sh::OFF_BK + kc * Sh::BCOL)) + 2 * k;
-          tc_mma_f16(tmem, smem_desc_sw128(smem_u32(sm + Sh::OFF_AHI + kc * Sh::ACOL)) + 2 * k, db, IDS,
-                     (kc | k) ? 1u : 0u);
-          tc_mma_f16(tmem, smem_desc_sw128(smem_u32(sm + Sh::OFF_ALO + kc * Sh::ACOL)) + 2 * k, db, IDS, 1u);
-        }
-      tc_commit(bar_s);
+    if (tid == 0 && more) {
+      if (pg + 3 < npages) stage_page(pg + 3);  // staging buffer (pg+1) & 1 has been read
+      issue_s(pg + 1);
     }
     __syncwarp();
-    mbar_wait(bar_s, pg & 1, s.err);
+    mbar_wait((pg & 1) ? bar_s1 : bar_s0, (pg >> 1) & 1, s.err);
     tc_fence_after();
 
-    float sc[64];
-#pragma unroll
-    for (int c0 = 0; c0 < 64; c0 += 16) tmem_ld_16(t_row + c0, sc + c0);
+    // this thread's 32 columns of the row
+    float sc[32];
+    tmem_ld_16(t_row + 64u * (uint32_t)(pg & 1) + 32u * half, sc);
+    tmem_ld_16(t_row + 64u * (uint32_t)(pg & 1) + 32u * half + 16u, sc + 16);
+    const int valid = min(64, last + 1 - pg * 64);
+    const int kb = pg * 64 + 32 * half;  // cache slot of this thread's first column
     float pm = -INFINITY;
+    if (row_ok && kb + 31 <= qslot && 32 * half + 31 < valid) {  // every key visible
 #pragma unroll
-    for (int c = 0; c < 64; ++c) {
-      const bool use = row_ok && c < valid && pg * 64 + c <= qslot;  // causal by cache slot
-      sc[c] = use ? sc[c] * scale : -INFINITY;
-      pm = fmaxf(pm, sc[c]);
+      for (int c = 0; c < 32; ++c) {
+        sc[c] *= scale;
+        pm = fmaxf(pm, sc[c]);
+      }
+    } else if (!row_ok || kb > qslot || 32 * half >= valid) {  // none visible
+#pragma unroll
+      for (int c = 0; c < 32; ++c) sc[c] = -INFINITY;
+    } else {  // the diagonal: causal by cache slot
+#pragma unroll
+      for (int c = 0; c < 32; ++c) {
+        const bool use = 32 * half + c < valid && kb + c <= qslot;
+        sc[c] = use ? sc[c] * scale : -INFINITY;
+        pm = fmaxf(pm, sc[c]);
+      }
     }
-    // lazy maximum: rescale only when it grows by more than 8 (warp-uniform TMEM access)
+    xch[half * 128 + row] = pm;
+    __syncthreads();
+    pm = fmaxf(pm, xch[(half ^ 1) * 128 + row]);
+    // lazy maximum: rescale only when it grows by more than 8 (warp-uniform TMEM access); both
+    // threads of a row take the same decision, each for its half of O and of the row sum
     const bool grow = pm > m_run + 8.f;
     const float cr = grow ? exp2f(m_run - pm) : 1.f;  // 0 when m_run was -inf
     if (__any_sync(0xffffffffu, grow) && pg > 0) {
 #pragma unroll
-      for (int c0 = 0; c0 < HD; c0 += 16) {
+      for (int c0 = 0; c0 < HD / 2; c0 += 16) {
         float o[16];
-        tmem_ld_16(t_row + 64 + c0, o);
+        tmem_ld_16(t_row + OCOL + (uint32_t)(half * (HD / 2) + c0), o);
 #pragma unroll
         for (int i = 0; i < 16; ++i) o[i] *= cr;
-        tmem_st_16(t_row + 64 + c0, o);
+        tmem_st_16(t_row + OCOL + (uint32_t)(half * (HD / 2) + c0), o);
       }
     }
     if (grow) {
       l_run *= cr;
       m_run = pm;
     }
-    uint32_t pk[32];
+    uint32_t pk[16];
     float psum = 0.f;
 #pragma unroll
-    for (int c = 0; c < 64; c += 2) {
-      const float p0 = sc[c] == -INFINITY ? 0.f : exp2f(sc[c] - m_run);
-      const float p1 = sc[c + 1] == -INFINITY ? 0.f : exp2f(sc[c + 1] - m_run);
+    for (int c = 0; c < 32; c += 2) {
+      const float p0 = sc[c] == -INFINITY ? 0.f : ex2_approx(sc[c] - m_run);
+      const float p1 = sc[c + 1] == -INFINITY ? 0.f : ex2_approx(sc[c + 1] - m_run);
+      psum += p0 + p1;
       pk[c / 2] = pack_bf16(p0, p1);
-      psum += __bfloat162float(__ushort_as_bfloat16((unsigned short)(pk[c / 2] & 0xFFFFu))) +
-              __bfloat162float(__ushort_as_bfloat16((unsigned short)(pk[c / 2] >> 16)));
     }
     l_run += psum;
 #pragma unroll
-    for (int q = 0; q < 8; ++q)
-      *reinterpret_cast<uint4*>(sm + Sh::OFF_P + sw128_off(tid, q)) =
+    for (int q = 0; q < 4; ++q)
+      *reinterpret_cast<uint4*>(sm + Sh::OFF_P + sw128_off(row, 4 * half + q)) =
           make_uint4(pk[4 * q], pk[4 * q + 1], pk[4 * q + 2], pk[4 * q + 3]);
     fence_proxy_async_smem();
     tc_fence_before();
     __syncthreads();
     if (tid == 0) {
       tc_fence_after();
+      const uint32_t bv = smem_u32(sm + Sh::OFF_BV + (pg & 1) * Sh::BV_BYTES);
 #pragma unroll
       for (int k = 0; k < 4; ++k)
-        tc_mma_f16(tmem + 64, smem_desc_sw128(smem_u32(sm + Sh::OFF_P)) + 2 * k,
-                   smem_desc_sw128(smem_u32(sm + Sh::OFF_BV)) + 2 * k, IDO, (pg > 0 || k > 0) ? 1u : 0u);
+        tc_mma_f16(tmem + OCOL, smem_desc_sw128(smem_u32(sm + Sh::OFF_P)) + 2 * k, smem_desc_sw128(bv) + 2 * k, IDO,
+                   (pg > 0 || k > 0) ? 1u : 0u);
       tc_commit(bar_o);
     }
     __syncwarp();
   }
   mbar_wait(bar_o, (npages - 1) & 1, s.err);
   tc_fence_after();
-  const float inv_l = l_run > 0.f ? 1.f / l_run : 0.f;
-  bf16* orow = O + (size_t)(first + q0 + qi) * md.q_dim + (kvh * G + g) * HD;
+  xch[half * 128 + row] = l_run;  // the two halves of each row sum
+  __syncthreads();
+  const float l_tot = l_run + xch[(half ^ 1) * 128 + row];
+  const float inv_l = l_tot > 0.f ? 1.f / l_tot : 0.f;
+  bf16* orow = O + (size_t)(first + q0 + qi) * md.q_dim + (kvh * G + g) * HD + half * (HD / 2);
 #pragma unroll
-  for (int c0 = 0; c0 < HD; c0 += 16) {
+  for (int c0 = 0; c0 < HD / 2; c0 += 16) {
     float o[16];
-    tmem_ld_16(t_row + 64 + c0, o);
+    tmem_ld_16(t_row + OCOL + (uint32_t)(half * (HD / 2) + c0), o);
     if (row_ok) {
       uint32_t w[8];
 #pragma unroll
