@@ -55,22 +55,27 @@ constexpr int TC_STAGES = 4;  // deepest operand ring; a launch uses min(4, k-ti
 
 // Dynamic shared memory of one CTA: the operand ring (reused after the main loop
 // for the cluster epilogue's fp32 partial tile [NT columns][128 features]), the
-// mbarriers and TMEM slot, and one int4 of per-column information per token.
+// mbarriers and TMEM slot, and per token column one int4 of information, one
+// float norm factor and four per-warp partial sums of squares.
 constexpr int tc_ring_bytes(int nt, int stages) { return stages * (TC_BM * TC_BK * 2 + nt * TC_BK * 2); }
 constexpr int tc_red_bytes(int nt) { return TC_BM * nt * 4; }
 constexpr int tc_body_bytes(int nt, int stages) {
   return tc_ring_bytes(nt, stages) > tc_red_bytes(nt) ? tc_ring_bytes(nt, stages) : tc_red_bytes(nt);
 }
 constexpr int tc_smem_bytes(int nt, int stages) {
-  return 1024 /*align slack*/ + tc_body_bytes(nt, stages) + 256 /*barriers, tmem slot*/ + nt * 16;
+  return 1024 /*align slack*/ + tc_body_bytes(nt, stages) + 256 /*barriers, tmem slot*/ + nt * (16 + 4 + 16);
 }
 
 // Second half of a cluster epilogue. Every CTA of the cluster has staged its
 // fp32 partial tile [NT columns][128 features] at `red`; this CTA sums the
 // partners' tiles over its share of the token columns through distributed
 // shared memory and finishes them according to the mode. `ci[c]` holds what
-// the mode needs per token column c: the residual row (RESID, in .w), or the
-// page, slot in page and position of the token's new cache entry (QKV).
+// the mode needs per token column c: for RESID the gate offset (.x), the next
+// norm's conditioning offset (.y), the column of the next operand (.z, -1:
+// none) and the residual row (.w, ~row for a row whose residual stays); for
+// QKV the page, slot in page and position of the token's new cache entry.
+// `scale[c]` is the column's RMSNorm factor when the operand arrives unscaled
+// (split norm), and `ssp` [4][NT] holds per-warp sums of squares (RESID).
 constexpr int CL_MAX = 8;  // largest cluster (split-K factor) of the cluster epilogues
 
 // Sums over the cluster of the staged values at feature f, columns c..c+3
@@ -92,12 +97,23 @@ __device__ __forceinline__ void cluster_sum4(const uint32_t* pb, int S, int f, i
   }
 }
 
-template <int NT>
-__device__ void cluster_epilogue(const GemmArgs& a, float* red, int4* ci, int m0, int n, int tok0) {
-  const int S = a.splits;
-  const int rank = (int)cluster_ctarank();
+// Columns of a cluster rank's share whose residual values the split-norm
+// epilogue takes from registers loaded before the main loop's end.
+constexpr int HPRE = 8;
+
+// The token columns [c0, c1) this CTA finishes in a cluster epilogue.
+__device__ __forceinline__ void cluster_cols(int n, int S, int& c0, int& c1) {
   const int per = (n + S - 1) / S;
-  const int c0 = rank * per, c1 = min(n, c0 + per);
+  c0 = (int)cluster_ctarank() * per;
+  c1 = min(n, c0 + per);
+}
+
+template <int NT>
+__device__ void cluster_epilogue(const GemmArgs& a, float* red, int4* ci, const float* scale, float* ssp,
+                                 const float (&hpre)[HPRE], int m0, int n, int tok0) {
+  const int S = a.splits;
+  int c0, c1;
+  cluster_cols(n, S, c0, c1);
   const int tid = threadIdx.x;
   uint32_t pb[CL_MAX];
   const uint32_t base = smem_u32(red);
@@ -106,17 +122,70 @@ __device__ void cluster_epilogue(const GemmArgs& a, float* red, int4* ci, int m0
 
   if (a.epi == EPI_CL_RESID) {
     const int col = m0 + tid;
-    if (col < a.N)
+    if (!a.xn) {
+      if (col < a.N)
+        for (int c = c0; c < c1; c += 4) {
+          float sm[4];
+          cluster_sum4(pb, S, tid, c, c1, sm);
+#pragma unroll
+          for (int q = 0; q < 4; ++q)
+            if (c + q < c1 && ci[c + q].w >= 0) {  // the only writer of this element
+              const float g = a.alpha.mod ? a.alpha.mod[ci[c + q].x + col] : 1.f;
+              atomicAdd(a.resid + (size_t)ci[c + q].w * a.ldr + col, g * sm[q]);
+            }
+        }
+      return;
+    }
+    // Split norm: the new residual value also feeds the next pre-norm. Every thread runs
+    // every column (features >= N count as 0) so the warp sums see full warps.
+    const bool fin = col < a.N;
+    const float gain = fin ? a.gain[col] : 0.f;
+    const int warp = tid >> 5, lane = tid & 31;
+    // column c (uniform over the CTA): h is its residual value before the update
+    auto finish = [&](int c, float h, float sm) {
+      const int4 e = ci[c];
+      if (fin && e.w >= 0) {  // the only writer of this element
+        const float g = a.alpha.mod ? a.alpha.mod[e.x + col] : 1.f;
+        h += g * sm;
+        a.resid[(size_t)e.w * a.ldr + col] = h;
+      }
+      if (e.z >= 0) {
+        if (fin) {
+          const float gm = a.gamma.mod ? 1.f + a.gamma.mod[e.y + col] : 1.f;
+          a.xn[(size_t)e.z * a.N + col] = __float2bfloat16_rn(h * gain * gm);
+        }
+        const float t = warp_sum(h * h);
+        if (lane == 0) ssp[warp * NT + c] = t;
+      }
+    };
+    if (c1 - c0 <= HPRE) {
+      float sm[HPRE];
+#pragma unroll
+      for (int q = 0; q < HPRE; q += 4) cluster_sum4(pb, S, tid, c0 + q, c1, sm + q);
+#pragma unroll
+      for (int q = 0; q < HPRE; ++q)
+        if (c0 + q < c1) finish(c0 + q, hpre[q], sm[q]);
+    } else {
       for (int c = c0; c < c1; c += 4) {
+        float hv[4];
+#pragma unroll
+        for (int q = 0; q < 4; ++q) {
+          const int w = (c + q < c1) ? ci[c + q].w : -1;
+          hv[q] = (fin && c + q < c1) ? a.resid[(size_t)(w >= 0 ? w : ~w) * a.ldr + col] : 0.f;
+        }
         float sm[4];
         cluster_sum4(pb, S, tid, c, c1, sm);
 #pragma unroll
         for (int q = 0; q < 4; ++q)
-          if (c + q < c1 && ci[c + q].w >= 0) {  // the only writer of this element
-            const float g = a.alpha.mod ? a.alpha.mod[ci[c + q].x + col] : 1.f;
-            atomicAdd(a.resid + (size_t)ci[c + q].w * a.ldr + col, g * sm[q]);
-          }
+          if (c + q < c1) finish(c + q, hv[q], sm[q]);
       }
+    }
+    __syncthreads();
+    for (int c = c0 + tid; c < c1; c += blockDim.x) {
+      const int dst = ci[c].z;
+      if (dst >= 0)
+        a.ss_out[(size_t)dst * a.ldss + m0 / TC_BM] = ssp[c] + ssp[NT + c] + ssp[2 * NT + c] + ssp[3 * NT + c];
+    }
     return;
   }
   if (a.epi == EPI_CL_SWIGLU) {
@@ -128,9 +197,12 @@ __device__ void cluster_epilogue(const GemmArgs& a, float* red, int4* ci, int m0
         cluster_sum4(pb, S, tid + 64, c, c1, u);
 #pragma unroll
         for (int q = 0; q < 4; ++q)
-          if (c + q < c1)
+          if (c + q < c1) {
+            const float f = a.ss_in ? scale[c + q] : 1.f;
+            const float gq = g[q] * f;
             reinterpret_cast<bf16*>(a.U)[(size_t)(tok0 + c + q) * a.md.ff + gf] =
-                __float2bfloat16_rn(g[q] / (1.f + expf(-g[q])) * u[q]);
+                __float2bfloat16_rn(gq / (1.f + expf(-gq)) * (u[q] * f));
+          }
       }
     return;
   }
@@ -176,6 +248,10 @@ __device__ void cluster_epilogue(const GemmArgs& a, float* red, int4* ci, int m0
       for (int q = 0; q < 4; ++q) {
         const int cc = c + q;
         if (cc >= c1) break;
+        if (a.ss_in) {
+          x0[q] *= scale[cc];
+          x1[q] *= scale[cc];
+        }
         const float r0 = x0[q] * csn[q].x - x1[q] * csn[q].y, r1 = x0[q] * csn[q].y + x1[q] * csn[q].x;
         if (is_q) {
           float* qo = a.Q + ((size_t)(tok0 + cc) * md.Hq + h) * hd;
@@ -204,7 +280,7 @@ __device__ void cluster_epilogue(const GemmArgs& a, float* red, int4* ci, int m0
         if (cc < c1 && ci[cc].x >= 0) {
           bf16* vp = pool + (size_t)ci[cc].x * md.page_elems + ((size_t)(a.j * 2 + 1) * md.Hkv + h) * ps * hd +
                      (size_t)ci[cc].y * hd;
-          vp[i] = __float2bfloat16_rn(x[q]);
+          vp[i] = __float2bfloat16_rn(a.ss_in ? x[q] * scale[cc] : x[q]);
         }
       }
     }
@@ -225,6 +301,8 @@ __global__ void __launch_bounds__(128) k_gemm_tc(const __grid_constant__ CUtenso
   uint64_t* bars = reinterpret_cast<uint64_t*>(smem + tc_body_bytes(NT, NS));
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 2 * TC_STAGES + 1);
   int4* colinfo = reinterpret_cast<int4*>(reinterpret_cast<uint8_t*>(bars) + 256);  // [NT]
+  float* colscale = reinterpret_cast<float*>(colinfo + NT);                          // [NT]
+  float* ssp = colscale + NT;                                                       // [4][NT]
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   // The token count comes from the plan kernel, which completed before this
@@ -294,17 +372,34 @@ __global__ void __launch_bounds__(128) k_gemm_tc(const __grid_constant__ CUtenso
     pdl_trigger();
     if (warp >= 2) {
       // idle during the main loop: fetch what the epilogue needs per token column
-      // (outputs of the plan kernel, read after the wait)
+      // (outputs of the plan kernel and of the preceding GEMM, read after the wait)
       for (int c = threadIdx.x - 64; c < n; c += 64) {
+        if (a.ss_in) {
+          // split norm: the column's factor from the producer's per-tile sums of squares
+          const float4* p4 = reinterpret_cast<const float4*>(a.ss_in + (size_t)(tok0 + c) * a.ldss);
+          float t = 0.f;
+#pragma unroll 4
+          for (int k = 0; k < a.ldss / 4; ++k) {
+            const float4 v = p4[k];
+            t += (v.x + v.y) + (v.z + v.w);
+          }
+          colscale[c] = rsqrtf(t / (float)a.K + a.norm_eps);
+        }
         if (a.epi == EPI_CL_QKV && !a.row_cslot) {
           colinfo[c] = a.s.rowinfo[a.r * a.md.max_batch + tok0 + c];
         } else if (a.epi == EPI_CL_RESID) {
-          // residual row; -1 for a row masked by the no-gather ablation (residual unchanged);
-          // with time/step conditioning, the offset of the row's gate vector in the table
+          // residual row, ~row for a row masked by the no-gather ablation (residual unchanged);
+          // with time/step conditioning, the offset of the row's gate vector in the table;
+          // with a split norm, the row's column in the next operand and its conditioning offset
+          const int row = a.idx ? a.idx[tok0 + c] : tok0 + c;
           const bool masked = a.act && !a.act[tok0 + c];
-          const int row = masked ? -1 : (a.idx ? a.idx[tok0 + c] : tok0 + c);
-          const int aoff = (a.alpha.mod && row >= 0) ? (int)(cond_row(a.alpha, row) - a.alpha.mod) : 0;
-          colinfo[c] = make_int4(aoff, 0, 0, row);
+          const int aoff = (a.alpha.mod && !masked) ? (int)(cond_row(a.alpha, row) - a.alpha.mod) : 0;
+          int goff = 0, dst = -1;
+          if (a.xn) {
+            dst = a.next_col ? a.next_col[row] : tok0 + c;
+            if (a.gamma.mod && dst >= 0) goff = (int)(cond_row(a.gamma, row) - a.gamma.mod);
+          }
+          colinfo[c] = make_int4(aoff, goff, dst, masked ? ~row : row);
         }
       }
     }
@@ -329,6 +424,25 @@ __global__ void __launch_bounds__(128) k_gemm_tc(const __grid_constant__ CUtenso
     }
   }
   __syncwarp();
+
+  // Split norm: load this thread's residual values (feature m0 + tid of its first
+  // HPRE columns) while the last MMAs drain; the epilogue updates them in place.
+  float hpre[HPRE];
+#pragma unroll
+  for (int q = 0; q < HPRE; ++q) hpre[q] = 0.f;
+  if (a.epi == EPI_CL_RESID && a.xn) {
+    int c0, c1;
+    cluster_cols(n, a.splits, c0, c1);
+    const int col = m0 + threadIdx.x;
+    if (c1 - c0 <= HPRE && col < a.N) {
+#pragma unroll
+      for (int q = 0; q < HPRE; ++q)
+        if (c0 + q < c1) {
+          const int row = a.idx ? a.idx[tok0 + c0 + q] : tok0 + c0 + q;
+          hpre[q] = a.resid[(size_t)row * a.ldr + col];
+        }
+    }
+  }
 
   // Epilogue: warp w holds output features m0 + 32w + lane; columns are token rows.
   bool ok = true;
@@ -356,7 +470,7 @@ __global__ void __launch_bounds__(128) k_gemm_tc(const __grid_constant__ CUtenso
     __syncthreads();
     if (warp == 0) tmem_dealloc(tmem, TMEM_COLS);
     cluster_sync_all();  // every partner's tile is staged
-    cluster_epilogue<NT>(a, red, colinfo, m0, n, tok0);
+    cluster_epilogue<NT>(a, red, colinfo, colscale, ssp, hpre, m0, n, tok0);
     __syncwarp();
     cluster_sync_all();  // partners have finished reading this CTA's tile
     return;

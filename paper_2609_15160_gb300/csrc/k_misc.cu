@@ -2,7 +2,9 @@
 //
 // k_norm_rows    gather + RMSNorm: X[k] = RMSNorm(H[idx[k]]) * gain for the
 //                rows of the active set (Eq. 6 followed by the pre-norm); with
-//                time/step conditioning the gain is scaled by (1 + gamma).
+//                time/step conditioning the gain is scaled by (1 + gamma). In
+//                split mode it writes H * gain unscaled plus the per-tile sums
+//                of squares, and the consuming GEMM applies the factor.
 // k_rope_table   (cos, sin) of every position x rotary frequency, built once.
 // k_rope_append  sums the split-K partials of the fused QKV projection (Eq. 9),
 //                rotates q and k at the token's original position, keeps q for
@@ -33,7 +35,8 @@ template <typename T>
 __global__ void __launch_bounds__(256) k_norm_rows(const float* __restrict__ H, int ldh, const int* __restrict__ idx,
                                                    const int* __restrict__ n_dev, int n_host,
                                                    const float* __restrict__ gain, int d, float eps,
-                                                   T* __restrict__ X, int ldx, CondArgs cg) {
+                                                   T* __restrict__ X, int ldx, CondArgs cg,
+                                                   float* __restrict__ ss_out, int ldss) {
   pdl_wait();
   pdl_trigger();
   const int k = blockIdx.x;
@@ -49,13 +52,21 @@ __global__ void __launch_bounds__(256) k_norm_rows(const float* __restrict__ H, 
 #pragma unroll
   for (int c = 0; c < 8; ++c) {
     const int i = threadIdx.x + c * blockDim.x;
+    float t = 0.f;
     if (i < d4) {
       v[c] = h4[i];
-      ss += v[c].x * v[c].x + v[c].y * v[c].y + v[c].z * v[c].z + v[c].w * v[c].w;
+      t = v[c].x * v[c].x + v[c].y * v[c].y + v[c].z * v[c].z + v[c].w * v[c].w;
     }
+    if (ss_out) {
+      // split norm: warp w of pass c holds features [128 (8c + w), +128), one tile of the partial sums
+      t = warp_sum(t);
+      if ((threadIdx.x & 31) == 0 && 4 * (c * blockDim.x + (threadIdx.x & ~31)) < d)
+        ss_out[(size_t)k * ldss + c * (blockDim.x >> 5) + (threadIdx.x >> 5)] = t;
+    }
+    ss += t;
   }
-  ss = block_sum(ss);
-  const float inv = rsqrtf(ss / (float)d + eps);
+  // split norm: the operand is written unscaled and the consumer applies the factor
+  const float inv = ss_out ? 1.f : rsqrtf(block_sum(ss) / (float)d + eps);
   T* xr = X + (size_t)k * ldx;
   // time/step conditioning: the gain is scaled by (1 + gamma) of the row's (depth, loop)
   const float4* c4 = cg.mod ? reinterpret_cast<const float4*>(cond_row(cg, src)) : nullptr;
@@ -77,13 +88,15 @@ __global__ void __launch_bounds__(256) k_norm_rows(const float* __restrict__ H, 
 }
 
 void launch_norm_rows(int dtype, const float* H, int ldh, const int* idx, const int* n_dev, int n_host, int rows_max,
-                      const float* gain, int d, float eps, void* X, int ldx, cudaStream_t st, const CondArgs& gamma) {
+                      const float* gain, int d, float eps, void* X, int ldx, cudaStream_t st, const CondArgs& gamma,
+                      float* ss_out) {
   if (rows_max <= 0) return;
   if (dtype == 1)
-    launch_k(k_norm_rows<bf16>, rows_max, 256, 0, st, H, ldh, idx, n_dev, n_host, gain, d, eps, (bf16*)X, ldx, gamma);
+    launch_k(k_norm_rows<bf16>, rows_max, 256, 0, st, H, ldh, idx, n_dev, n_host, gain, d, eps, (bf16*)X, ldx, gamma,
+             ss_out, split_norm_ldss(d));
   else
     launch_k(k_norm_rows<float>, rows_max, 256, 0, st, H, ldh, idx, n_dev, n_host, gain, d, eps, (float*)X, ldx,
-             gamma);
+             gamma, ss_out, split_norm_ldss(d));
 }
 
 // Rotary table: table[p][i] = (cos, sin)(p * theta_i), the angle formed and

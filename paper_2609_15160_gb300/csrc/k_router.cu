@@ -277,6 +277,7 @@ __global__ void __launch_bounds__(256) k_plan(ModelDims md, StepDev s, int B) {
       s.idx[r * maxB + k] = b;
       if (s.act) s.act[r * maxB + k] = active ? 1 : 0;
     }
+    if (s.col && b < B) s.col[r * maxB + b] = listed ? k : -1;
     // attention plan over the loop-r caches: an active token attends to its cache including its own
     // new entry; a masked row (no gather) to the entries already there. Every (token, kv head) item
     // spans ceil(keys / page) pages; items are laid out token-major in one flat page order

@@ -69,6 +69,9 @@ struct tlf_ctx {
   float* d_cond = nullptr;      // [J][M(M+1)/2][4][d] time/step modulation (conditioning only)
   int4* d_rowinfo = nullptr;    // [M][max_batch]
   int* d_act = nullptr;         // [M][max_batch]
+  int* d_col = nullptr;         // [M][max_batch] compact row of each residual row per loop
+  float* d_ss = nullptr;        // [max_batch][split_norm_ldss(d)] split RMSNorm partial sums of squares
+  bool split_norm = false;      // pre-norms split across the neighbouring GEMMs (tcgen05 path)
   std::vector<DeviceMat> wqkv, wo, wgu, wd;
   DeviceMat emb_mat;
 
@@ -529,6 +532,14 @@ static int create_impl(tlf_ctx* ctx, const tlf_weights* w) {
   if ((rc = dev_alloc(ctx, &ctx->d_attn_cnt, (size_t)B * md.Hkv * 4, "attention tickets"))) return rc;
   if ((rc = dev_alloc(ctx, &ctx->d_rowinfo, (size_t)M * B * sizeof(int4), "row info"))) return rc;
   if ((rc = dev_alloc(ctx, &ctx->d_act, (size_t)M * B * 4, "row masks"))) return rc;
+  if ((rc = dev_alloc(ctx, &ctx->d_col, (size_t)M * B * 4, "row columns"))) return rc;
+  if ((rc = dev_alloc(ctx, &ctx->d_ss, (size_t)split_norm_ldss(d) * B * 4, "norm partial sums"))) return rc;
+  CK(ctx, cudaMemset(ctx->d_ss, 0, (size_t)split_norm_ldss(d) * B * 4));
+  {
+    // TLF_NO_SPLIT_NORM=1 keeps every pre-norm a kernel of its own (comparison runs)
+    const char* e = getenv("TLF_NO_SPLIT_NORM");
+    ctx->split_norm = ctx->use_tc && !(e && e[0] == '1');
+  }
   CK(ctx, cudaMemset(ctx->d_attn_cnt, 0, (size_t)B * md.Hkv * 4));
   if ((rc = dev_alloc(ctx, &ctx->d_logits, (size_t)B * V * 4, "logits"))) return rc;
   if ((rc = dev_alloc(ctx, &ctx->d_err, 16, "error word"))) return rc;
@@ -553,7 +564,7 @@ extern "C" void tlf_destroy(tlf_ctx* ctx) {
     cudaDeviceSynchronize();
     auto f = [](void* p) { if (p) cudaFree(p); };
     f(ctx->d_emb); f(ctx->d_router_w); f(ctx->d_router_w1); f(ctx->d_router_b1); f(ctx->d_router_b); f(ctx->d_attn_norm); f(ctx->d_mlp_norm);
-    f(ctx->d_final_norm); f(ctx->d_inv_freq); f(ctx->d_rope); f(ctx->d_rowinfo); f(ctx->d_act); f(ctx->d_cond);
+    f(ctx->d_final_norm); f(ctx->d_inv_freq); f(ctx->d_rope); f(ctx->d_rowinfo); f(ctx->d_act); f(ctx->d_col); f(ctx->d_ss); f(ctx->d_cond);
     for (auto* v : {&ctx->wqkv, &ctx->wo, &ctx->wgu, &ctx->wd})
       for (auto& m : *v) f(m.ptr);
     f(ctx->d_pool); f(ctx->d_pos_table); f(ctx->d_page_table); f(ctx->d_len); f(ctx->d_upload);
@@ -730,6 +741,7 @@ static int enqueue_step(tlf_ctx* ctx, int B, bool need_logits, bool prof, cudaSt
   s.cnt = ctx->d_attn_cnt;
   s.rowinfo = ctx->d_rowinfo;
   s.act = ctx->d_act;
+  s.col = ctx->d_col;
   const PageUpdate* d_upd = reinterpret_cast<const PageUpdate*>(ctx->d_upload + 1 + 3 * B);
 
   ctx->last_launches = 0;
@@ -754,13 +766,24 @@ static int enqueue_step(tlf_ctx* ctx, int B, bool need_logits, bool prof, cudaSt
     // rows that do not run loop r but are computed anyway (no-gather ablation) keep their residual
     const int* act_r = md.ablation == TLF_ABLATION_NO_GATHER ? ctx->d_act + (size_t)r * maxB : nullptr;
     for (int j = 0; j < J; ++j) {
-      launch_norm_rows(md.dtype, ctx->d_H, md.d, idx_r, n_dev, 0, maxB, ctx->d_attn_norm + (size_t)j * md.d, md.d,
-                       md.eps, ctx->d_X, md.d, st, cond_args(ctx, s.m, r, j, 2));
-      mark(2);
+      // Split pre-norms: after the first, each norm's operand and partial sums are written by the
+      // residual epilogue before it and its factor applied by the GEMM after it.
+      const bool split = ctx->split_norm;
+      if (!split || (r == 0 && j == 0)) {
+        launch_norm_rows(md.dtype, ctx->d_H, md.d, idx_r, n_dev, 0, maxB, ctx->d_attn_norm + (size_t)j * md.d, md.d,
+                         md.eps, ctx->d_X, md.d, st, cond_args(ctx, s.m, r, j, 2), split ? ctx->d_ss : nullptr);
+        ++ctx->last_launches;
+        mark(2);
+      }
       GemmArgs a{};
       a.n_dev = n_dev;
       a.max_rows = maxB;
       a.splits = ctx->s_qkv;
+      if (split) {
+        a.ss_in = ctx->d_ss;
+        a.ldss = split_norm_ldss(md.d);
+        a.norm_eps = md.eps;
+      }
       if (ctx->use_tc) {
         // split-K reduction, RoPE and the K/V append run in the GEMM's cluster epilogue
         a.epi = EPI_CL_QKV;
@@ -793,15 +816,30 @@ static int enqueue_step(tlf_ctx* ctx, int B, bool need_logits, bool prof, cudaSt
       a.act = act_r;
       a.alpha = cond_args(ctx, s.m, r, j, 0);
       a.splits = ctx->s_o;
+      if (split) {  // the MLP pre-norm of this layer, same rows
+        a.xn = reinterpret_cast<bf16*>(ctx->d_X);
+        a.ss_out = ctx->d_ss;
+        a.ldss = split_norm_ldss(md.d);
+        a.gain = ctx->d_mlp_norm + (size_t)j * md.d;
+        a.gamma = cond_args(ctx, s.m, r, j, 3);
+      }
       gemm(ctx, ctx->wo[j], &ctx->map_O, ctx->d_O, md.q_dim, a, st);
       mark(6);
-      launch_norm_rows(md.dtype, ctx->d_H, md.d, idx_r, n_dev, 0, maxB, ctx->d_mlp_norm + (size_t)j * md.d, md.d,
-                       md.eps, ctx->d_X, md.d, st, cond_args(ctx, s.m, r, j, 3));
-      mark(7);
+      if (!split) {
+        launch_norm_rows(md.dtype, ctx->d_H, md.d, idx_r, n_dev, 0, maxB, ctx->d_mlp_norm + (size_t)j * md.d, md.d,
+                         md.eps, ctx->d_X, md.d, st, cond_args(ctx, s.m, r, j, 3));
+        ++ctx->last_launches;
+        mark(7);
+      }
       a = GemmArgs{};
       a.n_dev = n_dev;
       a.max_rows = maxB;
       a.splits = ctx->s_gu;
+      if (split) {
+        a.ss_in = ctx->d_ss;
+        a.ldss = split_norm_ldss(md.d);
+        a.norm_eps = md.eps;
+      }
       if (ctx->use_tc) {
         a.epi = EPI_CL_SWIGLU;  // SwiGLU in the cluster epilogue
         a.md = md;
@@ -827,9 +865,20 @@ static int enqueue_step(tlf_ctx* ctx, int B, bool need_logits, bool prof, cudaSt
       a.act = act_r;
       a.alpha = cond_args(ctx, s.m, r, j, 1);
       a.splits = ctx->s_d;
+      if (split && (j + 1 < J || r + 1 < M)) {
+        // the attention pre-norm of the next layer, or of layer 0 of loop r + 1 for the rows
+        // that continue (they move to their compact row of A_{r+1})
+        const int rn = j + 1 < J ? r : r + 1, jn = j + 1 < J ? j + 1 : 0;
+        a.xn = reinterpret_cast<bf16*>(ctx->d_X);
+        a.ss_out = ctx->d_ss;
+        a.ldss = split_norm_ldss(md.d);
+        a.gain = ctx->d_attn_norm + (size_t)jn * md.d;
+        a.gamma = cond_args(ctx, s.m, rn, jn, 2);
+        a.next_col = rn != r ? ctx->d_col + (size_t)rn * maxB : nullptr;
+      }
       gemm(ctx, ctx->wd[j], &ctx->map_U, ctx->d_U, md.ff, a, st);
       mark(10);
-      ctx->last_launches += 3;  // 2 norms and the attention (GEMMs counted in gemm())
+      ++ctx->last_launches;  // the attention (GEMMs counted in gemm(), norms where launched)
     }
   }
   launch_final(md, s, B, ctx->d_final_norm, ctx->d_Xf, st);

@@ -343,6 +343,8 @@ struct StepDev {
   int4* rowinfo;       // [M][maxB] per compact row k of A_r: {page, slot in page, position, 0} of the
                        // token's new loop-r cache entry (page -1 if the page table is corrupt);
                        // NULL for callers that only attend (the plan then writes no append targets)
+  int* col;            // [M][maxB] compact row of residual-stream row b in A_r, -1 if not listed
+                       // (inverse of idx; NULL: not written)
   // cache state
   int* len;            // [max_seqs][M] entries per (sequence, loop)
   int* page_table;     // [max_seqs][M][max_pages]
@@ -414,7 +416,24 @@ struct GemmArgs {
   const int* row_slot;
   const int* row_cslot;
   const int* row_pos;
+  // RMSNorm split across two GEMMs (EPI_CL_* decode path). The producer (a RESID
+  // epilogue) writes the next pre-norm's operand unscaled, xn[dst][f] =
+  // h[f] * gain[f] * (1 + gamma[f]), and per 128-feature tile t the partial sum
+  // ss[dst][t] = sum of h[f]^2 over the tile; the consumer (QKV or SwiGLU epilogue)
+  // scales column c of its product by rsqrt(sum_t ss[c][t] / K + eps), which is
+  // the row's RMSNorm factor moved past the (linear) projection. Rows of ss hold
+  // ldss = ceil(d / 128) rounded up to 4 entries, the padding kept at zero.
+  bf16* xn;                // producer: next operand [max_rows][N] (NULL: no fused norm)
+  float* ss_out;           // producer: [max_rows][ldss]
+  const float* gain;       // producer: the next norm's gain [N]
+  CondArgs gamma;          // producer: the next norm's conditioning (mod NULL: none)
+  const int* next_col;     // producer: column of residual row b in the next operand (NULL: same column)
+  const float* ss_in;      // consumer: [max_rows][ldss] (NULL: operand already normalised)
+  int ldss;
+  float norm_eps;
 };
+// Entries per row of the split-norm partial sums for model width d.
+inline int split_norm_ldss(int d) { return (((d + 127) / 128) + 3) / 4 * 4; }
 
 // ----------------------------------------------------------------------------
 // Launchers (host functions, one .cu file each)
@@ -431,7 +450,7 @@ void launch_plan(const ModelDims& md, const StepDev& s, int B, cudaStream_t st);
 
 void launch_norm_rows(int dtype, const float* H, int ldh, const int* idx, const int* n_dev, int n_host,
                       int rows_max, const float* gain, int d, float eps, void* X, int ldx, cudaStream_t st,
-                      const CondArgs& gamma = CondArgs{});
+                      const CondArgs& gamma = CondArgs{}, float* ss_out = nullptr);
 // Builds the conditioning table (see CondArgs) from the float32 weights on the device, in float64.
 int build_cond_table(const ModelDims& md, const float* t_w1, const float* t_b1, const float* t_w2, const float* t_b2,
                      const float* dt_w1, const float* dt_b1, const float* dt_w2, const float* dt_b2,

@@ -89,6 +89,13 @@ def test_c2_simt_gemm_path_matches_oracle(tlf):
     print(f"c2 simt worst {worst:.2e}")
 
 
+def test_c2_unsplit_norm_path_matches_oracle(tlf, monkeypatch):
+    """Every pre-norm as a kernel of its own (the tcgen05 path without the split norm)."""
+    monkeypatch.setenv("TLF_NO_SPLIT_NORM", "1")
+    worst, _ = _greedy_run(tlf, synth.get_config("c2"), steps=16)
+    print(f"c2 unsplit-norm worst {worst:.2e}")
+
+
 def _snapshot_run(T, wl, lengths, steps, sampled, seed=7, distinct=2, ablation="none"):
     """Sequences restored from synthetic cache snapshots, then decode steps of random tokens.
 
@@ -267,7 +274,10 @@ def test_wide_batch(tlf):
     _prefill_decode_compare(tlf, m, [3 + (b % 5) for b in range(160)], steps=2)
 
 
-def test_profile_counters(tlf):
+@pytest.mark.parametrize("split", [True, False])
+def test_profile_counters(tlf, monkeypatch, split):
+    if not split:
+        monkeypatch.setenv("TLF_NO_SPLIT_NORM", "1")
     m = _small()
     w = synth.make_weights(m)
     with tlf.Context(m, w, max_seqs=2, max_batch=2, max_seq_len=200) as ctx:
@@ -275,9 +285,10 @@ def test_profile_counters(tlf):
         ctx.set_profiling(True)
         _, loops, _ = ctx.decode_step([1, 2], [5, 6])
         ms, by, nl = ctx.last_step_profile()
-        # router, plan; per (loop, layer): 2 norms, QKV (+RoPE/append), attention, O, gate/up (+SwiGLU),
-        # down; final norm, LM head
-        assert ms > 0 and nl == 2 + m.max_loops * m.n_layers * 7 + 1 + 1
+        # router, plan; per (loop, layer): QKV (+RoPE/append), attention, O, gate/up (+SwiGLU), down and
+        # the two pre-norms, of which the split path launches only the step's first; final norm, LM head
+        per = 5 if split else 7
+        assert ms > 0 and nl == 2 + m.max_loops * m.n_layers * per + (1 if split else 0) + 1 + 1
         want = sum((ctx.cache_len(i, r)) * m.n_layers * 2 * m.n_kv_heads * m.head_dim * 2
                    for i, lp in zip([1, 2], loops) for r in range(1, lp + 1))
         assert abs(by - want) < 1e-6 * want
