@@ -122,6 +122,7 @@ __global__ void __launch_bounds__(ATT_THREADS) k_attn_decode(ModelDims md, StepD
   if (warp == ATT_WARPS) {
     // ---------------- producer warp ----------------
     if (lane == 0) {
+      const uint64_t kv_policy = l2_policy_evict_first();  // pages are read once per launch
       int k, h, g;
       locate(p0, k, h, g);
       int slot = s.slots[s.idx[r * maxB + k]];
@@ -144,8 +145,9 @@ __global__ void __launch_bounds__(ATT_THREADS) k_attn_decode(ModelDims md, StepD
           uint8_t* dst = ring + st * S::STAGE_BYTES;
           mbar_arrive_expect_tx(bar, 2 * bytes + (MASKED ? ATT_PS * 4 : 0));
           if (MASKED) bulk_g2s(smem_u32(mring + st * ATT_PS), s.pos_table + (size_t)page * ATT_PS, ATT_PS * 4, bar);
-          bulk_g2s(smem_u32(dst), pg + ((size_t)(j * 2 + 0) * Hkv + h) * ATT_PS * HD, bytes, bar);
-          bulk_g2s(smem_u32(dst + S::SEG_BYTES), pg + ((size_t)(j * 2 + 1) * Hkv + h) * ATT_PS * HD, bytes, bar);
+          bulk_g2s_hint(smem_u32(dst), pg + ((size_t)(j * 2 + 0) * Hkv + h) * ATT_PS * HD, bytes, bar, kv_policy);
+          bulk_g2s_hint(smem_u32(dst + S::SEG_BYTES), pg + ((size_t)(j * 2 + 1) * Hkv + h) * ATT_PS * HD, bytes, bar,
+                        kv_policy);
         }
         if (++g == pages_of(k)) {
           g = 0;

@@ -350,10 +350,13 @@ __global__ void __launch_bounds__(128) k_gemm_tc(const __grid_constant__ CUtenso
   if (warp == 0 && lane == 0) {
     // TMA producer. Weight tiles of the first stages go out before the wait on
     // the preceding kernels (weights are never written by them); token tiles after.
+    // decode reads each weight tile once per launch (streamed, evicted first); prefill's token
+    // tiles share them
+    const uint64_t w_policy = gridDim.z == 1 ? l2_policy_evict_first() : l2_policy_evict_normal();
     const int pre = nk < NS ? nk : NS;
     for (int i = 0; i < pre; ++i) {
       mbar_arrive_expect_tx(full(i), A_BYTES + B_BYTES);
-      tma_load_2d(smem_u32(sA + i * A_BYTES), &mapW, (kb0 + i) * TC_BK, m0, full(i));
+      tma_load_2d_hint(smem_u32(sA + i * A_BYTES), &mapW, (kb0 + i) * TC_BK, m0, full(i), w_policy);
     }
     pdl_wait();
     pdl_trigger();
@@ -364,7 +367,7 @@ __global__ void __launch_bounds__(128) k_gemm_tc(const __grid_constant__ CUtenso
       if (!mbar_wait(empty(st), ph ^ 1u, a.err)) break;
       mbar_arrive_expect_tx(full(st), A_BYTES + B_BYTES);
       const int kx = (kb0 + i) * TC_BK;
-      tma_load_2d(smem_u32(sA + st * A_BYTES), &mapW, kx, m0, full(st));
+      tma_load_2d_hint(smem_u32(sA + st * A_BYTES), &mapW, kx, m0, full(st), w_policy);
       tma_load_2d(smem_u32(sB + st * B_BYTES), &mapX, kx, tok0, full(st));
     }
   } else {
