@@ -188,16 +188,21 @@ __device__ void cluster_epilogue(const GemmArgs& a, float* red, int4* ci, const 
     }
     return;
   }
+  // With a pair of rows per output (gate and up, or the two halves of a rotary pair), the
+  // threads of the pair's upper row take the second half of the token columns.
+  const int cm = c0 + (c1 - c0 + 1) / 2;
   if (a.epi == EPI_CL_SWIGLU) {
-    const int gf = (m0 >> 1) + tid;  // 64 gate rows then 64 up rows per 128-row tile
-    if (tid < 64 && gf < a.md.ff)
-      for (int c = c0; c < c1; c += 4) {
+    const int f = tid & 63, hs = tid >> 6;
+    const int gf = (m0 >> 1) + f;  // 64 gate rows then 64 up rows per 128-row tile
+    const int ca = hs ? cm : c0, cb = hs ? c1 : cm;
+    if (gf < a.md.ff)
+      for (int c = ca; c < cb; c += 4) {
         float g[4], u[4];
-        cluster_sum4(pb, S, tid, c, c1, g);
-        cluster_sum4(pb, S, tid + 64, c, c1, u);
+        cluster_sum4(pb, S, f, c, cb, g);
+        cluster_sum4(pb, S, f + 64, c, cb, u);
 #pragma unroll
         for (int q = 0; q < 4; ++q)
-          if (c + q < c1) {
+          if (c + q < cb) {
             const float f = a.ss_in ? scale[c + q] : 1.f;
             const float gq = g[q] * f;
             reinterpret_cast<bf16*>(a.U)[(size_t)(tok0 + c + q) * a.md.ff + gf] =
@@ -234,20 +239,22 @@ __device__ void cluster_epilogue(const GemmArgs& a, float* red, int4* ci, const 
   if (gfeat < md.q_dim + md.kv_dim) {
     const bool is_q = gfeat < md.q_dim;
     const int fr = is_q ? gfeat : gfeat - md.q_dim;
-    const int h = fr / hd, i = fr % hd;
-    if (i >= half) return;  // the lower lane of the rotary pair handles both
-    for (int c = c0; c < c1; c += 4) {
+    const int h = fr / hd, hs = (fr % hd) >= half;
+    const int i = (fr % hd) - hs * half;   // rotary pair (i, i + half) of head h
+    const int tlo = tid - hs * half;       // tile row of the pair's lower element
+    const int ca = hs ? cm : c0, cb = hs ? c1 : cm;
+    for (int c = ca; c < cb; c += 4) {
       float2 csn[4];
 #pragma unroll
       for (int q = 0; q < 4; ++q)
-        csn[q] = (c + q < c1) ? a.rope[(size_t)ci[c + q].z * half + i] : make_float2(1.f, 0.f);
+        csn[q] = (c + q < cb) ? a.rope[(size_t)ci[c + q].z * half + i] : make_float2(1.f, 0.f);
       float x0[4], x1[4];
-      cluster_sum4(pb, S, tid, c, c1, x0);
-      cluster_sum4(pb, S, tid + half, c, c1, x1);
+      cluster_sum4(pb, S, tlo, c, cb, x0);
+      cluster_sum4(pb, S, tlo + half, c, cb, x1);
 #pragma unroll
       for (int q = 0; q < 4; ++q) {
         const int cc = c + q;
-        if (cc >= c1) break;
+        if (cc >= cb) break;
         if (a.ss_in) {
           x0[q] *= scale[cc];
           x1[q] *= scale[cc];
@@ -430,6 +437,7 @@ __global__ void __launch_bounds__(128) k_gemm_tc(const __grid_constant__ CUtenso
 
   // Split norm: load this thread's residual values (feature m0 + tid of its first
   // HPRE columns) while the last MMAs drain; the epilogue updates them in place.
+  // (Issued earlier, right after the wait, these loads measured slower.)
   float hpre[HPRE];
 #pragma unroll
   for (int q = 0; q < HPRE; ++q) hpre[q] = 0.f;
