@@ -69,8 +69,16 @@ __device__ __forceinline__ void consumer_sync() {
 template <typename T, int HD, int G, bool MASKED>
 __global__ void __launch_bounds__(ATT_THREADS) k_attn_decode(ModelDims md, StepDev s, int r, int j,
                                                              const float* __restrict__ Q, float* __restrict__ part,
-                                                             T* __restrict__ O, int* __restrict__ cnt) {
+                                                             T* __restrict__ O, int* __restrict__ cnt, bool o_lo) {
   using S = AttnShape<T, HD>;
+  // output element (token k, query head hq, dim e); with o_lo also the lo plane of the
+  // projection's two-term operand (bf16 of the rounding remainder, max_batch rows down)
+  auto store_o = [&](int k, int hq, int e, float val) {
+    const size_t at = (size_t)k * md.q_dim + (size_t)hq * HD + e;
+    const T hi = from_f32<T>(val);
+    O[at] = hi;
+    if (o_lo) O[(size_t)md.max_batch * md.q_dim + at] = from_f32<T>(val - to_f32(hi));
+  };
   constexpr int PSZ = G * (HD + 2);  // floats of one partial: per head, HD outputs then max and sum
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 127) & ~uintptr_t(127));
@@ -302,7 +310,7 @@ __global__ void __launch_bounds__(ATT_THREADS) k_attn_decode(ModelDims md, StepD
           l = fmaf(f, rw[HD + 1], l);
         }
         if (nparts == 1) {
-          O[(size_t)k * md.q_dim + (h * G + gg) * HD + e] = from_f32<T>(o / l);
+          store_o(k, h * G + gg, e, o / l);
         } else {
           my[gg * (HD + 2) + e] = o;
           if (e == 0) {
@@ -334,7 +342,7 @@ __global__ void __launch_bounds__(ATT_THREADS) k_attn_decode(ModelDims md, StepD
               o = fmaf(f, __ldcg(pp + e), o);
               l = fmaf(f, __ldcg(pp + HD + 1), l);
             }
-            O[(size_t)k * md.q_dim + (h * G + gg) * HD + e] = from_f32<T>(o / l);
+            store_o(k, h * G + gg, e, o / l);
           }
           if (tid == 0) cnt[item] = 0;  // ready for the next launch
         }
@@ -358,26 +366,27 @@ __global__ void __launch_bounds__(ATT_THREADS) k_attn_decode(ModelDims md, StepD
 
 template <typename T, int HD, int G, bool MASKED>
 static void attn_launch_v(const ModelDims& md, const StepDev& s, int r, int j, const float* Q, float* part, void* O,
-                          int* cnt, int grid, cudaStream_t st) {
+                          int* cnt, int grid, cudaStream_t st, bool o_lo) {
   static bool attr = false;
   constexpr int smem = attn_smem_bytes<T, HD, G, MASKED>();
   if (!attr) {
     cudaFuncSetAttribute(k_attn_decode<T, HD, G, MASKED>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
     attr = true;
   }
-  launch_k(k_attn_decode<T, HD, G, MASKED>, grid, ATT_THREADS, smem, st, md, s, r, j, Q, part, (T*)O, cnt);
+  launch_k(k_attn_decode<T, HD, G, MASKED>, grid, ATT_THREADS, smem, st, md, s, r, j, Q, part, (T*)O, cnt, o_lo);
 }
 
 template <typename T, int HD, int G>
 static void attn_launch(const ModelDims& md, const StepDev& s, int r, int j, const float* Q, float* part, void* O,
-                        int* cnt, int grid, cudaStream_t st) {
+                        int* cnt, int grid, cudaStream_t st, bool o_lo) {
+  o_lo = o_lo && std::is_same<T, bf16>::value;
   if constexpr (std::is_same<T, bf16>::value) {
     if (md.ablation == TLF_ABLATION_DENSE_CACHE) {
-      attn_launch_v<T, HD, G, true>(md, s, r, j, Q, part, O, cnt, grid, st);
+      attn_launch_v<T, HD, G, true>(md, s, r, j, Q, part, O, cnt, grid, st, o_lo);
       return;
     }
   }
-  attn_launch_v<T, HD, G, false>(md, s, r, j, Q, part, O, cnt, grid, st);
+  attn_launch_v<T, HD, G, false>(md, s, r, j, Q, part, O, cnt, grid, st, o_lo);
 }
 
 #define TLF_ATTN_DISPATCH(FN, ...)                                                              \
@@ -405,8 +414,8 @@ static void attn_launch(const ModelDims& md, const StepDev& s, int r, int j, con
   } while (0)
 
 void launch_attn_decode(const ModelDims& md, const StepDev& s, int r, int j, const float* Q, float* part, void* O,
-                        int* cnt, int grid, cudaStream_t st) {
-  TLF_ATTN_DISPATCH(attn_launch, md, s, r, j, Q, part, O, cnt, grid, st);
+                        int* cnt, int grid, cudaStream_t st, bool o_lo) {
+  TLF_ATTN_DISPATCH(attn_launch, md, s, r, j, Q, part, O, cnt, grid, st, o_lo);
 }
 
 // Resident CTAs: two per SM fit the ~104 KB ring of the largest head size.

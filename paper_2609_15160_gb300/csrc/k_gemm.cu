@@ -56,15 +56,34 @@ constexpr int TC_STAGES = 4;  // deepest operand ring; a launch uses min(4, k-ti
 // Dynamic shared memory of one CTA: the operand ring (reused after the main loop
 // for the cluster epilogue's fp32 partial tile [NT columns][128 features]), the
 // mbarriers and TMEM slot, and per token column one int4 of information, one
-// float norm factor and four per-warp partial sums of squares.
-constexpr int tc_ring_bytes(int nt, int stages) { return stages * (TC_BM * TC_BK * 2 + nt * TC_BK * 2); }
+// float norm factor and four per-warp partial sums of squares. With a two-term
+// operand (lo) a stage holds 2 x NT token rows.
+constexpr int tc_b_bytes(int nt, bool lo) { return (lo ? 2 : 1) * nt * TC_BK * 2; }
+constexpr int tc_ring_bytes(int nt, int stages, bool lo) { return stages * (TC_BM * TC_BK * 2 + tc_b_bytes(nt, lo)); }
 constexpr int tc_red_bytes(int nt) { return TC_BM * nt * 4; }
-constexpr int tc_body_bytes(int nt, int stages) {
-  return tc_ring_bytes(nt, stages) > tc_red_bytes(nt) ? tc_ring_bytes(nt, stages) : tc_red_bytes(nt);
+constexpr int tc_body_bytes(int nt, int stages, bool lo) {
+  return tc_ring_bytes(nt, stages, lo) > tc_red_bytes(nt) ? tc_ring_bytes(nt, stages, lo) : tc_red_bytes(nt);
 }
-constexpr int tc_smem_bytes(int nt, int stages) {
-  return 1024 /*align slack*/ + tc_body_bytes(nt, stages) + 256 /*barriers, tmem slot*/ + nt * (16 + 4 + 16);
+// TMEM columns of one CTA: the accumulator of 2 x NT columns (hi and lo halves) for
+// token tiles that may take a two-term operand, NT otherwise, at least 32.
+constexpr int tc_tmem_cols(int nt) {
+  return nt <= GEMM_LO_MAX_NT ? (2 * nt < 32 ? 32 : 2 * nt) : (nt < 32 ? 32 : nt);
 }
+// tcgen05.alloc blocks until columns are free, so the CTAs that shared memory lets
+// share an SM must fit in its 512 TMEM columns (otherwise clusters waiting for
+// partners could wait on each other): launches request at least this much.
+constexpr int SM_SMEM = 232448;  // shared memory per SM available to CTAs (227 KB + 1 KB per CTA)
+constexpr int tc_min_smem(int nt) { return SM_SMEM / (512 / tc_tmem_cols(nt) + 1) - 1024 + 1; }
+constexpr int tc_smem_bytes(int nt, int stages, bool lo) {
+  const int raw = 1024 /*align slack*/ + tc_body_bytes(nt, stages, lo) + 256 /*barriers, tmem slot*/ +
+                  nt * (16 + 4 + 16);
+  return raw > tc_min_smem(nt) ? raw : tc_min_smem(nt);
+}
+constexpr bool tmem_fits(int nt) {
+  return (SM_SMEM / (tc_smem_bytes(nt, 1, false) + 1024)) * tc_tmem_cols(nt) <= 512;
+}
+static_assert(tmem_fits(16) && tmem_fits(32) && tmem_fits(64) && tmem_fits(128) && tmem_fits(256),
+              "co-resident CTAs would oversubscribe TMEM");
 
 // Second half of a cluster epilogue. Every CTA of the cluster has staged its
 // fp32 partial tile [NT columns][128 features] at `red`; this CTA sums the
@@ -152,7 +171,10 @@ __device__ void cluster_epilogue(const GemmArgs& a, float* red, int4* ci, const 
       if (e.z >= 0) {
         if (fin) {
           const float gm = a.gamma.mod ? 1.f + a.gamma.mod[e.y + col] : 1.f;
-          a.xn[(size_t)e.z * a.N + col] = __float2bfloat16_rn(h * gain * gm);
+          const float y = h * gain * gm;
+          const bf16 yh = __float2bfloat16_rn(y);
+          a.xn[(size_t)e.z * a.N + col] = yh;
+          if (a.xn_lo) a.xn_lo[(size_t)e.z * a.N + col] = __float2bfloat16_rn(y - __bfloat162float(yh));
         }
         const float t = warp_sum(h * h);
         if (lane == 0) ssp[warp * NT + c] = t;
@@ -205,8 +227,11 @@ __device__ void cluster_epilogue(const GemmArgs& a, float* red, int4* ci, const 
           if (c + q < cb) {
             const float f = a.ss_in ? scale[c + q] : 1.f;
             const float gq = g[q] * f;
-            reinterpret_cast<bf16*>(a.U)[(size_t)(tok0 + c + q) * a.md.ff + gf] =
-                __float2bfloat16_rn(gq / (1.f + expf(-gq)) * (u[q] * f));
+            const float y = gq / (1.f + expf(-gq)) * (u[q] * f);
+            const bf16 yh = __float2bfloat16_rn(y);
+            const size_t at = (size_t)(tok0 + c + q) * a.md.ff + gf;
+            reinterpret_cast<bf16*>(a.U)[at] = yh;
+            if (a.U_lo) reinterpret_cast<bf16*>(a.U_lo)[at] = __float2bfloat16_rn(y - __bfloat162float(yh));
           }
       }
     return;
@@ -294,18 +319,30 @@ __device__ void cluster_epilogue(const GemmArgs& a, float* red, int4* ci, const 
   }
 }
 
+// 16 accumulator columns; with a two-term operand (lo_off > 0) plus the lo half lo_off columns on.
+__device__ __forceinline__ void tmem_ld_acc(uint32_t taddr, int lo_off, float* v) {
+  tmem_ld_16(taddr, v);
+  if (lo_off > 0) {
+    float w[16];
+    tmem_ld_16(taddr + (uint32_t)lo_off, w);
+#pragma unroll
+    for (int i = 0; i < 16; ++i) v[i] += w[i];
+  }
+}
+
 template <int NT>
 __global__ void __launch_bounds__(128) k_gemm_tc(const __grid_constant__ CUtensorMap mapW,
                                                  const __grid_constant__ CUtensorMap mapX, GemmArgs a) {
   constexpr int A_BYTES = TC_BM * TC_BK * 2;
-  constexpr int B_BYTES = NT * TC_BK * 2;
-  constexpr uint32_t TMEM_COLS = NT < 32 ? 32 : NT;
+  constexpr uint32_t TMEM_COLS = tc_tmem_cols(NT);
+  const bool lo = NT <= GEMM_LO_MAX_NT && a.blo > 0;  // two-term token operand
+  const int B_BYTES = tc_b_bytes(NT, lo);
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   const int NS = a.stages;  // 1..TC_STAGES
   uint8_t* sA = smem;
   uint8_t* sB = smem + NS * A_BYTES;
-  uint64_t* bars = reinterpret_cast<uint64_t*>(smem + tc_body_bytes(NT, NS));
+  uint64_t* bars = reinterpret_cast<uint64_t*>(smem + tc_body_bytes(NT, NS, lo));
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 2 * TC_STAGES + 1);
   int4* colinfo = reinterpret_cast<int4*>(reinterpret_cast<uint8_t*>(bars) + 256);  // [NT]
   float* colscale = reinterpret_cast<float*>(colinfo + NT);                          // [NT]
@@ -367,7 +404,12 @@ __global__ void __launch_bounds__(128) k_gemm_tc(const __grid_constant__ CUtenso
     }
     pdl_wait();
     pdl_trigger();
-    for (int i = 0; i < pre; ++i) tma_load_2d(smem_u32(sB + i * B_BYTES), &mapX, (kb0 + i) * TC_BK, tok0, full(i));
+    // token tiles; a two-term operand adds its lo plane (a.blo rows down) as rows NT..2NT-1
+    auto load_x = [&](int st, int kx) {
+      tma_load_2d(smem_u32(sB + st * B_BYTES), &mapX, kx, tok0, full(st));
+      if (lo) tma_load_2d(smem_u32(sB + st * B_BYTES + NT * TC_BK * 2), &mapX, kx, tok0 + a.blo, full(st));
+    };
+    for (int i = 0; i < pre; ++i) load_x(i, (kb0 + i) * TC_BK);
     for (int i = pre; i < nk; ++i) {
       const int st = i % NS;
       const uint32_t ph = (uint32_t)(i / NS) & 1u;
@@ -375,7 +417,7 @@ __global__ void __launch_bounds__(128) k_gemm_tc(const __grid_constant__ CUtenso
       mbar_arrive_expect_tx(full(st), A_BYTES + B_BYTES);
       const int kx = (kb0 + i) * TC_BK;
       tma_load_2d_hint(smem_u32(sA + st * A_BYTES), &mapW, kx, m0, full(st), w_policy);
-      tma_load_2d(smem_u32(sB + st * B_BYTES), &mapX, kx, tok0, full(st));
+      load_x(st, kx);
     }
   } else {
     pdl_wait();
@@ -417,7 +459,8 @@ __global__ void __launch_bounds__(128) k_gemm_tc(const __grid_constant__ CUtenso
   if (nk > 0) {
     if (warp == 1 && lane == 0) {
       // MMA issuer
-      const uint32_t idesc = idesc_bf16_f32(TC_BM, ncols);
+      // a two-term operand: MMA N covers the hi rows (NT) and the lo rows (NT)
+      const uint32_t idesc = idesc_bf16_f32(TC_BM, lo ? 2 * NT : ncols);
       for (int i = 0; i < nk; ++i) {
         const int st = i % NS;
         const uint32_t ph = (uint32_t)(i / NS) & 1u;
@@ -469,7 +512,7 @@ __global__ void __launch_bounds__(128) k_gemm_tc(const __grid_constant__ CUtenso
     for (int c0 = 0; c0 < ncols; c0 += 16) {
       float v[16];
       if (ok && nk > 0) {
-        tmem_ld_16(tmem + ((uint32_t)(warp * 32) << 16) + (uint32_t)c0, v);
+        tmem_ld_acc(tmem + ((uint32_t)(warp * 32) << 16) + (uint32_t)c0, lo ? NT : 0, v);
       } else {
 #pragma unroll
         for (int i = 0; i < 16; ++i) v[i] = 0.f;
@@ -491,7 +534,7 @@ __global__ void __launch_bounds__(128) k_gemm_tc(const __grid_constant__ CUtenso
     for (int c0 = 0; c0 < ncols; c0 += 16) {
       float v[16];
       if (nk > 0) {
-        tmem_ld_16(tmem + ((uint32_t)(warp * 32) << 16) + (uint32_t)c0, v);
+        tmem_ld_acc(tmem + ((uint32_t)(warp * 32) << 16) + (uint32_t)c0, lo ? NT : 0, v);
       } else {
 #pragma unroll
         for (int i = 0; i < 16; ++i) v[i] = 0.f;
@@ -516,28 +559,20 @@ int gemm_tc_stages(int K, int splits) {
   return per_cta < 1 ? 1 : (per_cta > TC_STAGES ? TC_STAGES : per_cta);
 }
 
-int gemm_tc_smem_bytes(int nt, int stages) { return tc_smem_bytes(nt, stages); }
+int gemm_tc_smem_bytes(int nt, int stages, bool lo) { return tc_smem_bytes(nt, stages, lo); }
 
-// Every CTA allocates max(32, NT) TMEM columns and tcgen05.alloc blocks until
-// columns are free, so as many CTAs as shared memory lets share an SM (the
-// smallest ring, of any kernel instance with the same NT) must fit in its 512
-// columns; otherwise clusters waiting for partners could wait on each other.
-constexpr int SM_SMEM = 232448;  // shared memory per SM available to CTAs (227 KB + 1 KB per CTA)
-constexpr bool tmem_fits(int nt) {
-  return (SM_SMEM / (tc_smem_bytes(nt, 1) + 1024)) * (nt < 32 ? 32 : nt) <= 512;
-}
-static_assert(tmem_fits(16) && tmem_fits(32) && tmem_fits(64) && tmem_fits(128) && tmem_fits(256),
-              "co-resident CTAs would oversubscribe TMEM");
 
 template <int NT>
 static void launch_tc_nt(const CUtensorMap* mapW, const CUtensorMap* mapX, GemmArgs a, cudaStream_t st) {
   static bool attr_set = false;
   if (!attr_set) {
-    cudaFuncSetAttribute(k_gemm_tc<NT>, cudaFuncAttributeMaxDynamicSharedMemorySize, tc_smem_bytes(NT, TC_STAGES));
+    cudaFuncSetAttribute(k_gemm_tc<NT>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                         tc_smem_bytes(NT, TC_STAGES, NT <= GEMM_LO_MAX_NT));
     attr_set = true;
   }
   a.stages = gemm_tc_stages(a.K, a.splits);
-  const int smem = tc_smem_bytes(NT, a.stages);
+  if (NT > GEMM_LO_MAX_NT) a.blo = 0;
+  const int smem = tc_smem_bytes(NT, a.stages, a.blo > 0);
   dim3 grid((a.N + TC_BM - 1) / TC_BM, a.splits, a.tok_tiles > 0 ? a.tok_tiles : 1);
   if (a.epi < EPI_CL_RESID) {
     launch_k(k_gemm_tc<NT>, grid, 128, smem, st, *mapW, *mapX, a);

@@ -36,7 +36,7 @@ __global__ void __launch_bounds__(256) k_norm_rows(const float* __restrict__ H, 
                                                    const int* __restrict__ n_dev, int n_host,
                                                    const float* __restrict__ gain, int d, float eps,
                                                    T* __restrict__ X, int ldx, CondArgs cg,
-                                                   float* __restrict__ ss_out, int ldss) {
+                                                   float* __restrict__ ss_out, int ldss, T* __restrict__ X_lo) {
   pdl_wait();
   pdl_trigger();
   const int k = blockIdx.x;
@@ -79,24 +79,27 @@ __global__ void __launch_bounds__(256) k_norm_rows(const float* __restrict__ H, 
         const float4 y = c4[i];
         g = make_float4(g.x * (1.f + y.x), g.y * (1.f + y.y), g.z * (1.f + y.z), g.w * (1.f + y.w));
       }
-      xr[4 * i + 0] = from_f32<T>(v[c].x * inv * g.x);
-      xr[4 * i + 1] = from_f32<T>(v[c].y * inv * g.y);
-      xr[4 * i + 2] = from_f32<T>(v[c].z * inv * g.z);
-      xr[4 * i + 3] = from_f32<T>(v[c].w * inv * g.w);
+      const float y[4] = {v[c].x * inv * g.x, v[c].y * inv * g.y, v[c].z * inv * g.z, v[c].w * inv * g.w};
+#pragma unroll
+      for (int e = 0; e < 4; ++e) {
+        const T hi = from_f32<T>(y[e]);
+        xr[4 * i + e] = hi;
+        if (X_lo) X_lo[(size_t)k * ldx + 4 * i + e] = from_f32<T>(y[e] - to_f32(hi));  // two-term operand
+      }
     }
   }
 }
 
 void launch_norm_rows(int dtype, const float* H, int ldh, const int* idx, const int* n_dev, int n_host, int rows_max,
                       const float* gain, int d, float eps, void* X, int ldx, cudaStream_t st, const CondArgs& gamma,
-                      float* ss_out) {
+                      float* ss_out, void* X_lo) {
   if (rows_max <= 0) return;
   if (dtype == 1)
     launch_k(k_norm_rows<bf16>, rows_max, 256, 0, st, H, ldh, idx, n_dev, n_host, gain, d, eps, (bf16*)X, ldx, gamma,
-             ss_out, split_norm_ldss(d));
+             ss_out, split_norm_ldss(d), (bf16*)X_lo);
   else
     launch_k(k_norm_rows<float>, rows_max, 256, 0, st, H, ldh, idx, n_dev, n_host, gain, d, eps, (float*)X, ldx,
-             gamma, ss_out, split_norm_ldss(d));
+             gamma, ss_out, split_norm_ldss(d), (float*)nullptr);
 }
 
 // Rotary table: table[p][i] = (cos, sin)(p * theta_i), the angle formed and

@@ -72,6 +72,7 @@ struct tlf_ctx {
   int* d_col = nullptr;         // [M][max_batch] compact row of each residual row per loop
   float* d_ss = nullptr;        // [max_batch][split_norm_ldss(d)] split RMSNorm partial sums of squares
   bool split_norm = false;      // pre-norms split across the neighbouring GEMMs (tcgen05 path)
+  bool operand_lo = false;      // X, O, U carry a lo plane (two-term GEMM operands, tcgen05 path)
   std::vector<DeviceMat> wqkv, wo, wgu, wd;
   DeviceMat emb_mat;
 
@@ -479,18 +480,25 @@ static int create_impl(tlf_ctx* ctx, const tlf_weights* w) {
   if ((rc = dev_alloc(ctx, &ctx->d_m, (size_t)B * 4, "m"))) return rc;
   if ((rc = dev_alloc(ctx, &ctx->d_margin, (size_t)B * 4, "margin"))) return rc;
   if ((rc = dev_alloc(ctx, &ctx->d_H, (size_t)B * d * 4, "H"))) return rc;
-  if ((rc = dev_alloc(ctx, &ctx->d_X, (size_t)B * d * eb, "X"))) return rc;
-  if ((rc = dev_alloc(ctx, &ctx->d_O, (size_t)B * md.q_dim * eb, "O"))) return rc;
-  if ((rc = dev_alloc(ctx, &ctx->d_U, (size_t)B * ff * eb, "U"))) return rc;
+  {
+    // two-term operands (hi + lo planes) where the token tile allows it; TLF_NO_OPERAND_LO=1
+    // keeps one bf16 plane (comparison runs)
+    const char* e = getenv("TLF_NO_OPERAND_LO");
+    ctx->operand_lo = ctx->use_tc && ctx->nt_max <= GEMM_LO_MAX_NT && !(e && e[0] == '1');
+  }
+  const int planes = ctx->operand_lo ? 2 : 1;
+  if ((rc = dev_alloc(ctx, &ctx->d_X, (size_t)planes * B * d * eb, "X"))) return rc;
+  if ((rc = dev_alloc(ctx, &ctx->d_O, (size_t)planes * B * md.q_dim * eb, "O"))) return rc;
+  if ((rc = dev_alloc(ctx, &ctx->d_U, (size_t)planes * B * ff * eb, "U"))) return rc;
   if ((rc = dev_alloc(ctx, &ctx->d_Xf, (size_t)B * d * eb, "Xf"))) return rc;
-  CK(ctx, cudaMemset(ctx->d_X, 0, (size_t)B * d * eb));
-  CK(ctx, cudaMemset(ctx->d_O, 0, (size_t)B * md.q_dim * eb));
-  CK(ctx, cudaMemset(ctx->d_U, 0, (size_t)B * ff * eb));
+  CK(ctx, cudaMemset(ctx->d_X, 0, (size_t)planes * B * d * eb));
+  CK(ctx, cudaMemset(ctx->d_O, 0, (size_t)planes * B * md.q_dim * eb));
+  CK(ctx, cudaMemset(ctx->d_U, 0, (size_t)planes * B * ff * eb));
   CK(ctx, cudaMemset(ctx->d_Xf, 0, (size_t)B * d * eb));
   if (ctx->use_tc) {
-    if (!make_map(&ctx->map_X, ctx->d_X, B, d, d, ctx->nt_max) ||
-        !make_map(&ctx->map_O, ctx->d_O, B, md.q_dim, md.q_dim, ctx->nt_max) ||
-        !make_map(&ctx->map_U, ctx->d_U, B, ff, ff, ctx->nt_max) ||
+    if (!make_map(&ctx->map_X, ctx->d_X, planes * B, d, d, ctx->nt_max) ||
+        !make_map(&ctx->map_O, ctx->d_O, planes * B, md.q_dim, md.q_dim, ctx->nt_max) ||
+        !make_map(&ctx->map_U, ctx->d_U, planes * B, ff, ff, ctx->nt_max) ||
         !make_map(&ctx->map_Xf, ctx->d_Xf, B, d, d, ctx->nt_max))
       return fail(ctx, TLF_ERR_CUDA, "cuTensorMapEncodeTiled failed for an activation buffer");
   }
@@ -501,7 +509,7 @@ static int create_impl(tlf_ctx* ctx, const tlf_weights* w) {
     auto pick = [&](int tiles, int K) {
       const int nkb = (K + 63) / 64;
       for (int S = std::min(8, nkb); S > 1; --S) {
-        const int bytes = gemm_tc_smem_bytes(ctx->nt_max, gemm_tc_stages(K, S));
+        const int bytes = gemm_tc_smem_bytes(ctx->nt_max, gemm_tc_stages(K, S), ctx->operand_lo);
         const int per_sm = std::min(16, 232448 / (bytes + 1024));
         if (10LL * tiles * S <= 9LL * per_sm * ctx->num_sms) return S;
       }
@@ -760,6 +768,11 @@ static int enqueue_step(tlf_ctx* ctx, int B, bool need_logits, bool prof, cudaSt
   launch_plan(md, s, B, st);
   mark(1);
   ctx->last_launches += 2;
+  // two-term GEMM operands: lo planes of X, U (and O, written by the attention kernel) sit
+  // max_batch rows below the hi planes
+  const int lo_rows = ctx->operand_lo ? maxB : 0;
+  void* x_lo = ctx->operand_lo ? static_cast<void*>(reinterpret_cast<bf16*>(ctx->d_X) + (size_t)maxB * md.d) : nullptr;
+  void* u_lo = ctx->operand_lo ? static_cast<void*>(reinterpret_cast<bf16*>(ctx->d_U) + (size_t)maxB * md.ff) : nullptr;
   for (int r = 0; r < M; ++r) {
     const int* n_dev = ctx->d_n + r;
     const int* idx_r = ctx->d_idx + (size_t)r * maxB;
@@ -771,7 +784,8 @@ static int enqueue_step(tlf_ctx* ctx, int B, bool need_logits, bool prof, cudaSt
       const bool split = ctx->split_norm;
       if (!split || (r == 0 && j == 0)) {
         launch_norm_rows(md.dtype, ctx->d_H, md.d, idx_r, n_dev, 0, maxB, ctx->d_attn_norm + (size_t)j * md.d, md.d,
-                         md.eps, ctx->d_X, md.d, st, cond_args(ctx, s.m, r, j, 2), split ? ctx->d_ss : nullptr);
+                         md.eps, ctx->d_X, md.d, st, cond_args(ctx, s.m, r, j, 2), split ? ctx->d_ss : nullptr,
+                         x_lo);
         ++ctx->last_launches;
         mark(2);
       }
@@ -779,6 +793,7 @@ static int enqueue_step(tlf_ctx* ctx, int B, bool need_logits, bool prof, cudaSt
       a.n_dev = n_dev;
       a.max_rows = maxB;
       a.splits = ctx->s_qkv;
+      a.blo = lo_rows;
       if (split) {
         a.ss_in = ctx->d_ss;
         a.ldss = split_norm_ldss(md.d);
@@ -804,7 +819,8 @@ static int enqueue_step(tlf_ctx* ctx, int B, bool need_logits, bool prof, cudaSt
         ++ctx->last_launches;
         mark(4);
       }
-      launch_attn_decode(md, s, r, j, ctx->d_Q, ctx->d_attn_part, ctx->d_O, ctx->d_attn_cnt, ctx->attn_grid, st);
+      launch_attn_decode(md, s, r, j, ctx->d_Q, ctx->d_attn_part, ctx->d_O, ctx->d_attn_cnt, ctx->attn_grid, st,
+                         ctx->operand_lo);
       mark(5);
       a = GemmArgs{};
       a.n_dev = n_dev;
@@ -816,8 +832,10 @@ static int enqueue_step(tlf_ctx* ctx, int B, bool need_logits, bool prof, cudaSt
       a.act = act_r;
       a.alpha = cond_args(ctx, s.m, r, j, 0);
       a.splits = ctx->s_o;
+      a.blo = lo_rows;
       if (split) {  // the MLP pre-norm of this layer, same rows
         a.xn = reinterpret_cast<bf16*>(ctx->d_X);
+        a.xn_lo = reinterpret_cast<bf16*>(x_lo);
         a.ss_out = ctx->d_ss;
         a.ldss = split_norm_ldss(md.d);
         a.gain = ctx->d_mlp_norm + (size_t)j * md.d;
@@ -827,7 +845,7 @@ static int enqueue_step(tlf_ctx* ctx, int B, bool need_logits, bool prof, cudaSt
       mark(6);
       if (!split) {
         launch_norm_rows(md.dtype, ctx->d_H, md.d, idx_r, n_dev, 0, maxB, ctx->d_mlp_norm + (size_t)j * md.d, md.d,
-                         md.eps, ctx->d_X, md.d, st, cond_args(ctx, s.m, r, j, 3));
+                         md.eps, ctx->d_X, md.d, st, cond_args(ctx, s.m, r, j, 3), nullptr, x_lo);
         ++ctx->last_launches;
         mark(7);
       }
@@ -835,6 +853,7 @@ static int enqueue_step(tlf_ctx* ctx, int B, bool need_logits, bool prof, cudaSt
       a.n_dev = n_dev;
       a.max_rows = maxB;
       a.splits = ctx->s_gu;
+      a.blo = lo_rows;
       if (split) {
         a.ss_in = ctx->d_ss;
         a.ldss = split_norm_ldss(md.d);
@@ -844,6 +863,7 @@ static int enqueue_step(tlf_ctx* ctx, int B, bool need_logits, bool prof, cudaSt
         a.epi = EPI_CL_SWIGLU;  // SwiGLU in the cluster epilogue
         a.md = md;
         a.U = ctx->d_U;
+        a.U_lo = u_lo;
         gemm(ctx, ctx->wgu[j], &ctx->map_X, ctx->d_X, md.d, a, st);
         mark(8);
       } else {
@@ -865,11 +885,13 @@ static int enqueue_step(tlf_ctx* ctx, int B, bool need_logits, bool prof, cudaSt
       a.act = act_r;
       a.alpha = cond_args(ctx, s.m, r, j, 1);
       a.splits = ctx->s_d;
+      a.blo = lo_rows;
       if (split && (j + 1 < J || r + 1 < M)) {
         // the attention pre-norm of the next layer, or of layer 0 of loop r + 1 for the rows
         // that continue (they move to their compact row of A_{r+1})
         const int rn = j + 1 < J ? r : r + 1, jn = j + 1 < J ? j + 1 : 0;
         a.xn = reinterpret_cast<bf16*>(ctx->d_X);
+        a.xn_lo = reinterpret_cast<bf16*>(x_lo);
         a.ss_out = ctx->d_ss;
         a.ldss = split_norm_ldss(md.d);
         a.gain = ctx->d_attn_norm + (size_t)jn * md.d;

@@ -465,6 +465,13 @@ struct GemmArgs {
   const float* ss_in;      // consumer: [max_rows][ldss] (NULL: operand already normalised)
   int ldss;
   float norm_eps;
+  // Two-term bf16 operand (tcgen05 decode path, token tiles <= 64). An activation v is
+  // stored as hi = bf16(v) and lo = bf16(v - hi) in two planes of one buffer, lo at row
+  // offset max_rows, and the GEMM multiplies both (MMA N = 2 x tile, halves summed in the
+  // epilogue), so the operand keeps about 16 significant bits instead of 8.
+  int blo;                 // consumer: row offset of the token operand's lo plane (0: one plane)
+  bf16* xn_lo;             // producer (split norm): lo plane of xn (NULL: none)
+  void* U_lo;              // EPI_CL_SWIGLU: lo plane of U (NULL: none)
 };
 // Entries per row of the split-norm partial sums for model width d.
 inline int split_norm_ldss(int d) { return (((d + 127) / 128) + 3) / 4 * 4; }
@@ -484,7 +491,7 @@ void launch_plan(const ModelDims& md, const StepDev& s, int B, cudaStream_t st);
 
 void launch_norm_rows(int dtype, const float* H, int ldh, const int* idx, const int* n_dev, int n_host,
                       int rows_max, const float* gain, int d, float eps, void* X, int ldx, cudaStream_t st,
-                      const CondArgs& gamma = CondArgs{}, float* ss_out = nullptr);
+                      const CondArgs& gamma = CondArgs{}, float* ss_out = nullptr, void* X_lo = nullptr);
 // Builds the conditioning table (see CondArgs) from the float32 weights on the device, in float64.
 int build_cond_table(const ModelDims& md, const float* t_w1, const float* t_b1, const float* t_w2, const float* t_b2,
                      const float* dt_w1, const float* dt_b1, const float* dt_w2, const float* dt_b2,
@@ -497,13 +504,17 @@ int gemm_tc_max_nt();
 // operand-ring depth of a tcgen05 GEMM whose CTAs each reduce ceil(ceil(K/64)/splits) k-tiles,
 // and the dynamic shared memory one CTA of token tile nt then needs
 int gemm_tc_stages(int K, int splits);
-int gemm_tc_smem_bytes(int nt, int stages);
+int gemm_tc_smem_bytes(int nt, int stages, bool lo = false);
+// largest token tile whose GEMMs take a two-term (hi + lo) operand
+constexpr int GEMM_LO_MAX_NT = 64;
 
 void launch_rope_table(const ModelDims& md, const double* inv_freq, float2* table, cudaStream_t st);
 void launch_rope_append(const ModelDims& md, const StepDev& s, int r, int j, const float* part, int splits,
                         float* Q, const float2* rope, cudaStream_t st);
+// o_lo (bf16 models): also write O's lo plane (bf16 of the rounding remainder) at row offset
+// max_batch, the two-term operand of the output projection
 void launch_attn_decode(const ModelDims& md, const StepDev& s, int r, int j, const float* Q, float* part, void* O,
-                        int* cnt, int grid, cudaStream_t st);
+                        int* cnt, int grid, cudaStream_t st, bool o_lo = false);
 int attn_decode_grid(const ModelDims& md, int num_sms);
 size_t attn_partial_floats(const ModelDims& md, int grid);
 

@@ -96,6 +96,13 @@ def test_c2_unsplit_norm_path_matches_oracle(tlf, monkeypatch):
     print(f"c2 unsplit-norm worst {worst:.2e}")
 
 
+def test_one_plane_operand_path_matches_oracle(tlf, monkeypatch):
+    """The tcgen05 path with single bf16 GEMM operands (no lo planes)."""
+    monkeypatch.setenv("TLF_NO_OPERAND_LO", "1")
+    worst, _ = _greedy_run(tlf, synth.get_config("c2"), steps=16)
+    print(f"c2 one-plane worst {worst:.2e}")
+
+
 def _snapshot_run(T, wl, lengths, steps, sampled, seed=7, distinct=2, ablation="none"):
     """Sequences restored from synthetic cache snapshots, then decode steps of random tokens.
 
@@ -159,6 +166,15 @@ def test_c3_full_size_sampled_parity(tlf):
     lengths = np.full(wl.batch, wl.prompt_len[0])
     worst, forced = _snapshot_run(tlf, wl, lengths, steps=4, sampled=[0, 37])
     print(f"c3 worst {worst:.2e} forced {forced}")
+
+
+def test_two_term_operands_keep_deep_models_precise(tlf):
+    """C3 (8 loops x 4 layers) at 16 tokens: with hi + lo bf16 GEMM operands the logits stay
+    within 5e-3 of the float64 oracle, a quarter of the 2e-2 bound (one bf16 plane: about 1.9e-2)."""
+    wl = synth.get_config("c3")
+    lengths = np.full(16, wl.prompt_len[0])
+    worst, _ = _snapshot_run(tlf, wl.with_batch(16), lengths, steps=3, sampled=[0, 5])
+    assert worst < 5e-3, worst
 
 
 def test_c4_full_size_sampled_parity(tlf):
