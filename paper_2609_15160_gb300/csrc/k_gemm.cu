@@ -100,7 +100,13 @@ constexpr int CL_MAX = 8;  // largest cluster (split-K factor) of the cluster ep
 // Sums over the cluster of the staged values at feature f, columns c..c+3
 // (columns >= c1 give 0). All partner loads of the four columns are issued
 // before any is used.
-__device__ __forceinline__ void cluster_sum4(const uint32_t* pb, int S, int f, int c, int c1, float out[4]) {
+__device__ __forceinline__ void cluster_sum4(const uint32_t* pb, const float* red, int S, int f, int c, int c1,
+                                             float out[4]) {
+  if (S == 1) {  // one split (prefill): the CTA's own staged tile, plain shared loads
+#pragma unroll
+    for (int q = 0; q < 4; ++q) out[q] = (c + q < c1) ? red[(c + q) * 128 + f] : 0.f;
+    return;
+  }
   float v[CL_MAX][4];
 #pragma unroll
   for (int p = 0; p < CL_MAX; ++p)
@@ -145,7 +151,7 @@ __device__ void cluster_epilogue(const GemmArgs& a, float* red, int4* ci, const 
       if (col < a.N)
         for (int c = c0; c < c1; c += 4) {
           float sm[4];
-          cluster_sum4(pb, S, tid, c, c1, sm);
+          cluster_sum4(pb, red, S, tid, c, c1, sm);
 #pragma unroll
           for (int q = 0; q < 4; ++q)
             if (c + q < c1 && ci[c + q].w >= 0) {  // the only writer of this element
@@ -183,7 +189,7 @@ __device__ void cluster_epilogue(const GemmArgs& a, float* red, int4* ci, const 
     if (c1 - c0 <= HPRE) {
       float sm[HPRE];
 #pragma unroll
-      for (int q = 0; q < HPRE; q += 4) cluster_sum4(pb, S, tid, c0 + q, c1, sm + q);
+      for (int q = 0; q < HPRE; q += 4) cluster_sum4(pb, red, S, tid, c0 + q, c1, sm + q);
 #pragma unroll
       for (int q = 0; q < HPRE; ++q)
         if (c0 + q < c1) finish(c0 + q, hpre[q], sm[q]);
@@ -196,7 +202,7 @@ __device__ void cluster_epilogue(const GemmArgs& a, float* red, int4* ci, const 
           hv[q] = (fin && c + q < c1) ? a.resid[(size_t)(w >= 0 ? w : ~w) * a.ldr + col] : 0.f;
         }
         float sm[4];
-        cluster_sum4(pb, S, tid, c, c1, sm);
+        cluster_sum4(pb, red, S, tid, c, c1, sm);
 #pragma unroll
         for (int q = 0; q < 4; ++q)
           if (c + q < c1) finish(c + q, hv[q], sm[q]);
@@ -220,8 +226,8 @@ __device__ void cluster_epilogue(const GemmArgs& a, float* red, int4* ci, const 
     if (gf < a.md.ff)
       for (int c = ca; c < cb; c += 4) {
         float g[4], u[4];
-        cluster_sum4(pb, S, f, c, cb, g);
-        cluster_sum4(pb, S, f + 64, c, cb, u);
+        cluster_sum4(pb, red, S, f, c, cb, g);
+        cluster_sum4(pb, red, S, f + 64, c, cb, u);
 #pragma unroll
         for (int q = 0; q < 4; ++q)
           if (c + q < cb) {
@@ -274,8 +280,8 @@ __device__ void cluster_epilogue(const GemmArgs& a, float* red, int4* ci, const 
       for (int q = 0; q < 4; ++q)
         csn[q] = (c + q < cb) ? a.rope[(size_t)ci[c + q].z * half + i] : make_float2(1.f, 0.f);
       float x0[4], x1[4];
-      cluster_sum4(pb, S, tlo, c, cb, x0);
-      cluster_sum4(pb, S, tlo + half, c, cb, x1);
+      cluster_sum4(pb, red, S, tlo, c, cb, x0);
+      cluster_sum4(pb, red, S, tlo + half, c, cb, x1);
 #pragma unroll
       for (int q = 0; q < 4; ++q) {
         const int cc = c + q;
@@ -305,7 +311,7 @@ __device__ void cluster_epilogue(const GemmArgs& a, float* red, int4* ci, const 
     const int h = fr / hd, i = fr % hd;
     for (int c = c0; c < c1; c += 4) {
       float x[4];
-      cluster_sum4(pb, S, tid, c, c1, x);
+      cluster_sum4(pb, red, S, tid, c, c1, x);
 #pragma unroll
       for (int q = 0; q < 4; ++q) {
         const int cc = c + q;
