@@ -60,9 +60,11 @@ constexpr int TC_STAGES = 4;  // deepest operand ring; a launch uses min(4, k-ti
 // operand (lo) a stage holds 2 x NT token rows.
 constexpr int tc_b_bytes(int nt, bool lo) { return (lo ? 2 : 1) * nt * TC_BK * 2; }
 constexpr int tc_ring_bytes(int nt, int stages, bool lo) { return stages * (TC_BM * TC_BK * 2 + tc_b_bytes(nt, lo)); }
-constexpr int tc_red_bytes(int nt) { return TC_BM * nt * 4; }
-constexpr int tc_body_bytes(int nt, int stages, bool lo) {
-  return tc_ring_bytes(nt, stages, lo) > tc_red_bytes(nt) ? tc_ring_bytes(nt, stages, lo) : tc_red_bytes(nt);
+constexpr int tc_red_bytes(int red_cols) { return TC_BM * red_cols * 4; }
+// red_cols: token columns of the staged fp32 tile (nt, or the window of a one-split epilogue)
+constexpr int tc_body_bytes(int nt, int stages, bool lo, int red_cols) {
+  return tc_ring_bytes(nt, stages, lo) > tc_red_bytes(red_cols) ? tc_ring_bytes(nt, stages, lo)
+                                                                : tc_red_bytes(red_cols);
 }
 // TMEM columns of one CTA: the accumulator of 2 x NT columns (hi and lo halves) for
 // token tiles that may take a two-term operand, NT otherwise, at least 32.
@@ -74,8 +76,9 @@ constexpr int tc_tmem_cols(int nt) {
 // partners could wait on each other): launches request at least this much.
 constexpr int SM_SMEM = 232448;  // shared memory per SM available to CTAs (227 KB + 1 KB per CTA)
 constexpr int tc_min_smem(int nt) { return SM_SMEM / (512 / tc_tmem_cols(nt) + 1) - 1024 + 1; }
-constexpr int tc_smem_bytes(int nt, int stages, bool lo) {
-  const int raw = 1024 /*align slack*/ + tc_body_bytes(nt, stages, lo) + 256 /*barriers, tmem slot*/ +
+constexpr int tc_smem_bytes(int nt, int stages, bool lo, int red_cols = 0) {
+  const int raw = 1024 /*align slack*/ + tc_body_bytes(nt, stages, lo, red_cols > 0 ? red_cols : nt) +
+                  256 /*barriers, tmem slot*/ +
                   nt * (16 + 4 + 16);
   return raw > tc_min_smem(nt) ? raw : tc_min_smem(nt);
 }
@@ -100,11 +103,13 @@ constexpr int CL_MAX = 8;  // largest cluster (split-K factor) of the cluster ep
 // Sums over the cluster of the staged values at feature f, columns c..c+3
 // (columns >= c1 give 0). All partner loads of the four columns are issued
 // before any is used.
-__device__ __forceinline__ void cluster_sum4(const uint32_t* pb, const float* red, int S, int f, int c, int c1,
-                                             float out[4]) {
-  if (S == 1) {  // one split (prefill): the CTA's own staged tile, plain shared loads
+// With one split (prefill) the CTA's own staged tile is read with plain shared loads; it may
+// hold the window of columns starting at roff.
+__device__ __forceinline__ void cluster_sum4(const uint32_t* pb, const float* red, int roff, int S, int f, int c,
+                                             int c1, float out[4]) {
+  if (S == 1) {
 #pragma unroll
-    for (int q = 0; q < 4; ++q) out[q] = (c + q < c1) ? red[(c + q) * 128 + f] : 0.f;
+    for (int q = 0; q < 4; ++q) out[q] = (c + q < c1) ? red[(c + q - roff) * 128 + f] : 0.f;
     return;
   }
   float v[CL_MAX][4];
@@ -135,10 +140,13 @@ __device__ __forceinline__ void cluster_cols(int n, int S, int& c0, int& c1) {
 
 template <int NT>
 __device__ void cluster_epilogue(const GemmArgs& a, float* red, int4* ci, const float* scale, float* ssp,
-                                 const float (&hpre)[HPRE], int m0, int n, int tok0) {
+                                 const float (&hpre)[HPRE], int m0, int n, int tok0, int cw0, int cw1) {
   const int S = a.splits;
   int c0, c1;
   cluster_cols(n, S, c0, c1);
+  // columns of this pass: the CTA's share within the staged window [cw0, cw1) (the whole share
+  // unless a one-split epilogue stages in windows; the split-norm path is never windowed)
+  const int w0 = c0 > cw0 ? c0 : cw0, w1 = c1 < cw1 ? c1 : cw1;
   const int tid = threadIdx.x;
   uint32_t pb[CL_MAX];
   const uint32_t base = smem_u32(red);
@@ -149,12 +157,12 @@ __device__ void cluster_epilogue(const GemmArgs& a, float* red, int4* ci, const 
     const int col = m0 + tid;
     if (!a.xn) {
       if (col < a.N)
-        for (int c = c0; c < c1; c += 4) {
+        for (int c = w0; c < w1; c += 4) {
           float sm[4];
-          cluster_sum4(pb, red, S, tid, c, c1, sm);
+          cluster_sum4(pb, red, cw0, S, tid, c, w1, sm);
 #pragma unroll
           for (int q = 0; q < 4; ++q)
-            if (c + q < c1 && ci[c + q].w >= 0) {  // the only writer of this element
+            if (c + q < w1 && ci[c + q].w >= 0) {  // the only writer of this element
               const float g = a.alpha.mod ? a.alpha.mod[ci[c + q].x + col] : 1.f;
               atomicAdd(a.resid + (size_t)ci[c + q].w * a.ldr + col, g * sm[q]);
             }
@@ -189,7 +197,7 @@ __device__ void cluster_epilogue(const GemmArgs& a, float* red, int4* ci, const 
     if (c1 - c0 <= HPRE) {
       float sm[HPRE];
 #pragma unroll
-      for (int q = 0; q < HPRE; q += 4) cluster_sum4(pb, red, S, tid, c0 + q, c1, sm + q);
+      for (int q = 0; q < HPRE; q += 4) cluster_sum4(pb, red, 0, S, tid, c0 + q, c1, sm + q);
 #pragma unroll
       for (int q = 0; q < HPRE; ++q)
         if (c0 + q < c1) finish(c0 + q, hpre[q], sm[q]);
@@ -202,7 +210,7 @@ __device__ void cluster_epilogue(const GemmArgs& a, float* red, int4* ci, const 
           hv[q] = (fin && c + q < c1) ? a.resid[(size_t)(w >= 0 ? w : ~w) * a.ldr + col] : 0.f;
         }
         float sm[4];
-        cluster_sum4(pb, red, S, tid, c, c1, sm);
+        cluster_sum4(pb, red, 0, S, tid, c, c1, sm);
 #pragma unroll
         for (int q = 0; q < 4; ++q)
           if (c + q < c1) finish(c + q, hv[q], sm[q]);
@@ -218,16 +226,16 @@ __device__ void cluster_epilogue(const GemmArgs& a, float* red, int4* ci, const 
   }
   // With a pair of rows per output (gate and up, or the two halves of a rotary pair), the
   // threads of the pair's upper row take the second half of the token columns.
-  const int cm = c0 + (c1 - c0 + 1) / 2;
+  const int cm = w0 + (w1 - w0 + 1) / 2;
   if (a.epi == EPI_CL_SWIGLU) {
     const int f = tid & 63, hs = tid >> 6;
     const int gf = (m0 >> 1) + f;  // 64 gate rows then 64 up rows per 128-row tile
-    const int ca = hs ? cm : c0, cb = hs ? c1 : cm;
+    const int ca = hs ? cm : w0, cb = hs ? w1 : cm;
     if (gf < a.md.ff)
       for (int c = ca; c < cb; c += 4) {
         float g[4], u[4];
-        cluster_sum4(pb, red, S, f, c, cb, g);
-        cluster_sum4(pb, red, S, f + 64, c, cb, u);
+        cluster_sum4(pb, red, cw0, S, f, c, cb, g);
+        cluster_sum4(pb, red, cw0, S, f + 64, c, cb, u);
 #pragma unroll
         for (int q = 0; q < 4; ++q)
           if (c + q < cb) {
@@ -246,8 +254,9 @@ __device__ void cluster_epilogue(const GemmArgs& a, float* red, int4* ci, const 
   const ModelDims& md = a.md;
   const StepDev& s = a.s;
   const int ps = md.page_size, hd = md.hd, half = hd / 2;
-  if (a.row_cslot) {
-    // prefill: sequence slot, cache slot and position of each row from the prefill plan
+  if (a.row_cslot && cw0 == 0) {
+    // prefill: sequence slot, cache slot and position of each row from the prefill plan (once, in
+    // the first window)
     for (int c = c0 + tid; c < c1; c += blockDim.x) {
       const int row = tok0 + c;
       const int slot = a.row_slot[row], L = a.row_cslot[row];
@@ -273,15 +282,15 @@ __device__ void cluster_epilogue(const GemmArgs& a, float* red, int4* ci, const 
     const int h = fr / hd, hs = (fr % hd) >= half;
     const int i = (fr % hd) - hs * half;   // rotary pair (i, i + half) of head h
     const int tlo = tid - hs * half;       // tile row of the pair's lower element
-    const int ca = hs ? cm : c0, cb = hs ? c1 : cm;
+    const int ca = hs ? cm : w0, cb = hs ? w1 : cm;
     for (int c = ca; c < cb; c += 4) {
       float2 csn[4];
 #pragma unroll
       for (int q = 0; q < 4; ++q)
         csn[q] = (c + q < cb) ? a.rope[(size_t)ci[c + q].z * half + i] : make_float2(1.f, 0.f);
       float x0[4], x1[4];
-      cluster_sum4(pb, red, S, tlo, c, cb, x0);
-      cluster_sum4(pb, red, S, tlo + half, c, cb, x1);
+      cluster_sum4(pb, red, cw0, S, tlo, c, cb, x0);
+      cluster_sum4(pb, red, cw0, S, tlo + half, c, cb, x1);
 #pragma unroll
       for (int q = 0; q < 4; ++q) {
         const int cc = c + q;
@@ -309,13 +318,13 @@ __device__ void cluster_epilogue(const GemmArgs& a, float* red, int4* ci, const 
   } else {
     const int fr = gfeat - md.q_dim - md.kv_dim;
     const int h = fr / hd, i = fr % hd;
-    for (int c = c0; c < c1; c += 4) {
+    for (int c = w0; c < w1; c += 4) {
       float x[4];
-      cluster_sum4(pb, red, S, tid, c, c1, x);
+      cluster_sum4(pb, red, cw0, S, tid, c, w1, x);
 #pragma unroll
       for (int q = 0; q < 4; ++q) {
         const int cc = c + q;
-        if (cc < c1 && ci[cc].x >= 0) {
+        if (cc < w1 && ci[cc].x >= 0) {
           bf16* vp = pool + (size_t)ci[cc].x * md.page_elems + ((size_t)(a.j * 2 + 1) * md.Hkv + h) * ps * hd +
                      (size_t)ci[cc].y * hd;
           vp[i] = __float2bfloat16_rn(a.ss_in ? x[q] * scale[cc] : x[q]);
@@ -348,7 +357,9 @@ __global__ void __launch_bounds__(128) k_gemm_tc(const __grid_constant__ CUtenso
   const int NS = a.stages;  // 1..TC_STAGES
   uint8_t* sA = smem;
   uint8_t* sB = smem + NS * A_BYTES;
-  uint64_t* bars = reinterpret_cast<uint64_t*>(smem + tc_body_bytes(NT, NS, lo));
+  // one-split epilogues may stage the tile in windows of red_window columns (smaller smem)
+  const int RW = (a.red_window > 0 && a.splits == 1 && a.red_window < NT) ? a.red_window : NT;
+  uint64_t* bars = reinterpret_cast<uint64_t*>(smem + tc_body_bytes(NT, NS, lo, RW));
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 2 * TC_STAGES + 1);
   int4* colinfo = reinterpret_cast<int4*>(reinterpret_cast<uint8_t*>(bars) + 256);  // [NT]
   float* colscale = reinterpret_cast<float*>(colinfo + NT);                          // [NT]
@@ -515,24 +526,28 @@ __global__ void __launch_bounds__(128) k_gemm_tc(const __grid_constant__ CUtenso
     // tile layout [column][128 features]: a warp's partner reads are 128 contiguous bytes
     float* red = reinterpret_cast<float*>(smem);
     const int f = warp * 32 + lane;
-    for (int c0 = 0; c0 < ncols; c0 += 16) {
-      float v[16];
-      if (ok && nk > 0) {
-        tmem_ld_acc(tmem + ((uint32_t)(warp * 32) << 16) + (uint32_t)c0, lo ? NT : 0, v);
-      } else {
+    for (int w = 0; w < ncols; w += RW) {  // one pass unless a one-split tile is staged in windows
+      const int wend = w + RW < ncols ? w + RW : ncols;
+      if (w > 0) __syncthreads();  // every thread is done with the previous window
+      for (int c0 = w; c0 < wend; c0 += 16) {
+        float v[16];
+        if (ok && nk > 0) {
+          tmem_ld_acc(tmem + ((uint32_t)(warp * 32) << 16) + (uint32_t)c0, lo ? NT : 0, v);
+        } else {
 #pragma unroll
-        for (int i = 0; i < 16; ++i) v[i] = 0.f;
+          for (int i = 0; i < 16; ++i) v[i] = 0.f;
+        }
+#pragma unroll
+        for (int i = 0; i < 16; ++i) red[(c0 - w + i) * 128 + f] = v[i];
       }
-#pragma unroll
-      for (int i = 0; i < 16; ++i) red[(c0 + i) * 128 + f] = v[i];
+      tc_fence_before();
+      __syncthreads();
+      if (wend == ncols && warp == 0) tmem_dealloc(tmem, TMEM_COLS);
+      cluster_sync_all();  // every partner's tile is staged
+      cluster_epilogue<NT>(a, red, colinfo, colscale, ssp, hpre, m0, n, tok0, w, w + RW);
+      __syncwarp();
+      cluster_sync_all();  // partners have finished reading this CTA's tile
     }
-    tc_fence_before();
-    __syncthreads();
-    if (warp == 0) tmem_dealloc(tmem, TMEM_COLS);
-    cluster_sync_all();  // every partner's tile is staged
-    cluster_epilogue<NT>(a, red, colinfo, colscale, ssp, hpre, m0, n, tok0);
-    __syncwarp();
-    cluster_sync_all();  // partners have finished reading this CTA's tile
     return;
   }
   if (ok) {
@@ -578,7 +593,16 @@ static void launch_tc_nt(const CUtensorMap* mapW, const CUtensorMap* mapX, GemmA
   }
   a.stages = gemm_tc_stages(a.K, a.splits);
   if (NT > GEMM_LO_MAX_NT) a.blo = 0;
-  const int smem = tc_smem_bytes(NT, a.stages, a.blo > 0);
+  int red_cols = NT;
+  if (a.red_window > 0 && a.splits == 1 && a.red_window < NT) {
+    // windowed one-split epilogue: with a 2-stage ring two CTAs share an SM, so one CTA's
+    // epilogue overlaps the other's main loop
+    red_cols = a.red_window;
+    if (a.stages > 2) a.stages = 2;
+  } else {
+    a.red_window = 0;
+  }
+  const int smem = tc_smem_bytes(NT, a.stages, a.blo > 0, red_cols);
   dim3 grid((a.N + TC_BM - 1) / TC_BM, a.splits, a.tok_tiles > 0 ? a.tok_tiles : 1);
   if (a.epi < EPI_CL_RESID) {
     launch_k(k_gemm_tc<NT>, grid, 128, smem, st, *mapW, *mapX, a);

@@ -1108,6 +1108,7 @@ static void gemm_pf(tlf_ctx* ctx, const DeviceMat& W, const CUtensorMap* xmap, G
   a.K = W.K;
   a.err = ctx->d_err;
   a.splits = 1;
+  a.red_window = 128;  // stage 128 of the 256 token columns at a time: two CTAs per SM
   a.max_rows = ctx->pf_C;
   a.tok_tiles = ctx->pf_C / 256;
   launch_gemm_tc(&W.map, xmap, 256, a, st);

@@ -470,6 +470,7 @@ struct GemmArgs {
   // offset max_rows, and the GEMM multiplies both (MMA N = 2 x tile, halves summed in the
   // epilogue), so the operand keeps about 16 significant bits instead of 8.
   int blo;                 // consumer: row offset of the token operand's lo plane (0: one plane)
+  int red_window;          // cluster epilogues with one split: token columns staged per pass (0: all)
   bf16* xn_lo;             // producer (split norm): lo plane of xn (NULL: none)
   void* U_lo;              // EPI_CL_SWIGLU: lo plane of U (NULL: none)
 };
