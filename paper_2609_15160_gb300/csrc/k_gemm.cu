@@ -1,34 +1,46 @@
 // Dense projections of the shared block on the compacted tokens (Eq. 6, 9):
 // Y[row][o] = sum_k X[row][k] * W[o][k] for the n rows of the active set.
 //
-// k_gemm_tc (bf16): tcgen05 tensor-core GEMM. Operand roles are swapped so
-// that the weight tile fills the 128-row MMA dimension and the n <= 256 tokens
-// form the N dimension (decode has few tokens and many output features).
-// Warp 0 lane 0 streams 128x64 weight tiles and NTx64 token tiles into a
-// 4-stage shared-memory ring with 2-D TMA (128-byte swizzle); warp 1 lane 0
-// issues tcgen05.mma (M=128, N=round16(n), K=16) accumulating in TMEM and
-// releases each stage with tcgen05.commit; then all four warps read the
-// accumulator with tcgen05.ld (warp w owns TMEM lanes 32w..32w+31 = output
-// features) and run the epilogue. Split-K over gridDim.y keeps enough CTAs
-// in flight to stream the weights at HBM speed.
+// k_gemm_tc (bf16): tcgen05 tensor-core GEMM. Operand roles are swapped so that
+// the weight tile fills the 128-row MMA dimension and the n <= 256 tokens form
+// the N dimension (decode has few tokens and many output features).
+// - Warp 0 lane 0 streams 128x64 weight tiles and NTx64 token tiles into a
+//   shared-memory ring of 1-4 stages with 2-D TMA (128-byte swizzle).
+// - The first stages' weight tiles go out before the grid-dependency wait
+//   (programmatic dependent launch). Decode weights carry an L2 evict-first
+//   hint, because each tile is read once per launch.
+// - Warp 1 lane 0 issues tcgen05.mma (M=128, K=16) accumulating in TMEM and
+//   releases each stage with tcgen05.commit.
+// - All four warps then read the accumulator with tcgen05.ld (warp w owns TMEM
+//   lanes 32w..32w+31 = output features) and run the epilogue. Split-K over
+//   gridDim.y keeps enough CTAs in flight to stream the weights at HBM speed.
+// Two-term operands (decode, token tiles <= 64): the token operand arrives as
+// bf16 hi and lo planes, loaded as one B tile of 2 x NT rows; the MMA runs with
+// N = 2 x NT and the epilogue adds the two accumulator halves.
 //
 // k_gemm_simt: CUDA-core tiled GEMM with the same epilogues, for float32
 // models (tcgen05 has no exact float32 mode) and as a second GPU path.
 //
-// Epilogues of the bf16 decode path (cluster epilogues): the S split-K CTAs
-// of one 128-feature tile are launched as a (1, S, 1) thread-block cluster.
-// Each stages its partial tile in shared memory; after a cluster barrier
-// every CTA sums a 1/S share of the tile over the cluster through distributed
-// shared memory (fixed order, so results are deterministic) and finishes it:
-// residual add + scatter into the float32 stream H[idx[row]] (Eq. 7, one
-// writer per element), RoPE on q and k at the token's original position with
-// k and v appended to its loop-r page (Eq. 9, 11), or silu(gate) * up
-// (SwiGLU; gate and up rows interleave per 64-feature tile so one tile holds
-// both halves). No partial sum leaves the chip and no separate kernel runs.
+// Cluster epilogues: the S split-K CTAs of one 128-feature tile are launched as
+// a (1, S, 1) thread-block cluster. Each stages its partial tile in shared
+// memory. After a cluster barrier every CTA sums a 1/S share of the tile over
+// the cluster through distributed shared memory, in a fixed order, so results
+// are deterministic. It then finishes the share in one of three ways:
+// - residual add + scatter into the float32 stream H[idx[row]] (Eq. 7, one
+//   writer per element); with a split pre-norm it also writes the next GEMM's
+//   unscaled operand and per-tile sums of squares;
+// - RoPE on q and k at the token's original position, with k and v appended to
+//   its loop-r page (Eq. 9, 11);
+// - silu(gate) * up (SwiGLU; gate and up rows interleave per 64-feature tile, so
+//   one tile holds both halves).
+// No partial sum leaves the chip and no separate kernel runs. Consumers of a
+// split pre-norm scale each token column by its RMSNorm factor first. With one
+// split (prefill) the CTA reads its own tile with plain shared loads and may
+// stage it in 128-column windows, so two CTAs share an SM.
 //
-// Other epilogues (SIMT path, prefill, LM head): split-K partial sums to a
-// buffer consumed by k_rope_append / k_swiglu, atomic residual add + scatter,
-// or a plain float32 store (logits).
+// Other epilogues (SIMT path, LM head): split-K partial sums to a buffer
+// consumed by k_rope_append / k_swiglu, atomic residual add + scatter, or a
+// plain float32 store (logits).
 #include "tlf_internal.cuh"
 
 namespace tlf {
