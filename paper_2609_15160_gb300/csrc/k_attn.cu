@@ -18,7 +18,9 @@
 // the lengths, and streams them without draining its pipeline at item
 // boundaries. A producer warp copies the K and V segments of each page (64
 // keys of one kv head, contiguous and 16-byte aligned) into an NST-deep
-// shared-memory ring with 1-D bulk TMA copies that complete on mbarriers; the
+// shared-memory ring with 1-D bulk TMA copies that complete on mbarriers. The
+// copies carry an L2 evict-first hint: each page is read once per launch, and the
+// hint keeps the step's small reused buffers resident in L2. The
 // eight consumer warps split every page, release the stage on a per-stage
 // mbarrier, and keep an online-softmax state (running max, sum, output slice)
 // in float32 for the G query heads of the kv head (grouped-query attention),
@@ -26,10 +28,12 @@
 // Scores are in base 2 (q pre-scaled by log2(e)/sqrt(hd)).
 //
 // When a CTA finishes its part of an item it merges its warps. An item that
-// lies inside one CTA's range is written out directly; otherwise each
+// lies inside one CTA's range is written out directly. Otherwise each
 // contributing CTA stores a partial (max, sum, output) and takes a ticket with
 // an atomic counter, and the CTA that takes the last ticket merges the
-// partials and writes the output (no CTA ever waits for another).
+// partials and writes the output (no CTA ever waits for another). On the
+// tcgen05 decode path the output also gets its lo plane, bf16(o - bf16(o)): the
+// output projection then takes a two-term operand.
 #include <type_traits>
 
 #include "tlf_internal.cuh"
