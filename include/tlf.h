@@ -174,7 +174,21 @@ int64_t tlf_page_bytes(const tlf_config* cfg);
 /* Create a context: validate cfg, copy the weights to the current CUDA
  * device, allocate the KV page pool and step workspaces. *out receives the
  * context (NULL on failure). On failure the message is available through
- * tlf_last_error(NULL) on the same thread. */
+ * tlf_last_error(NULL) on the same thread.
+ *
+ * Environment switches select equivalent comparison paths, each covered by
+ * the GPU tests. The first two change only how kernels are launched, and the
+ * results are bit-identical; the last two change rounding, within the logits
+ * tolerance.
+ *   TLF_NO_GRAPH=1       launch each step's kernels directly instead of
+ *                        replaying a captured CUDA graph (read here)
+ *   TLF_NO_PDL=1         plain stream order instead of programmatic
+ *                        dependent launch (read when the library loads)
+ *   TLF_NO_SPLIT_NORM=1  every decode pre-norm as a kernel of its own instead
+ *                        of split across the neighbouring GEMMs (read here)
+ *   TLF_NO_OPERAND_LO=1  one bf16 plane for the decode GEMMs' activation
+ *                        operands instead of hi + lo (two-term) planes (read
+ *                        here) */
 int tlf_create(const tlf_config* cfg, const tlf_weights* w, tlf_ctx** out);
 
 /* Free every device and host resource of the context. NULL is a no-op. */

@@ -584,8 +584,6 @@ __global__ void __launch_bounds__(128) k_gemm_tc(const __grid_constant__ CUtenso
   if (warp == 0) tmem_dealloc(tmem, TMEM_COLS);
 }
 
-int gemm_tc_max_nt() { return 256; }
-
 int gemm_tc_stages(int K, int splits) {
   const int nkb = (K + TC_BK - 1) / TC_BK;
   const int per_cta = (nkb + splits - 1) / splits;

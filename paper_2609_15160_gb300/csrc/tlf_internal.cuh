@@ -501,7 +501,6 @@ int build_cond_table(const ModelDims& md, const float* t_w1, const float* t_b1, 
 void launch_gemm_simt(int dtype, const void* W, const void* X, int ldx, const GemmArgs& a, cudaStream_t st);
 void launch_gemm_tc(const CUtensorMap* mapW, const CUtensorMap* mapX, int nt_max, const GemmArgs& a,
                     cudaStream_t st);
-int gemm_tc_max_nt();
 // operand-ring depth of a tcgen05 GEMM whose CTAs each reduce ceil(ceil(K/64)/splits) k-tiles,
 // and the dynamic shared memory one CTA of token tile nt then needs
 int gemm_tc_stages(int K, int splits);

@@ -378,6 +378,50 @@ def test_decode_step_is_deterministic(tlf):
         np.testing.assert_array_equal(a, b)
 
 
+# Launch mechanics only (no arithmetic changes): the direct-launch and plain stream-order paths
+# must reproduce the graph-replayed, programmatic-dependent-launch step bit for bit.
+_LAUNCH_RUN = """
+import sys
+import numpy as np
+sys.path.insert(0, {root!r})
+from paper_2609_15160_gb300 import synth, tlf as T
+m = synth.ModelConfig(vocab=300, d_model=256, n_heads=4, n_kv_heads=2, head_dim=64, n_layers=2, ffn_hidden=320,
+                      max_loops=3, dtype="bf16", depth_probs=(0.3, 0.3, 0.4))
+w = synth.make_weights(m)
+rng = np.random.default_rng(5)
+prompts = [rng.integers(0, m.vocab, size=n).astype(np.int32) for n in (90, 33, 64)]
+steps = [rng.integers(0, m.vocab, size=3).astype(np.int32) for _ in range(4)]
+out = []
+with T.Context(m, w, max_seqs=3, max_batch=3, max_seq_len=200) as ctx:
+    lg, _ = ctx.prefill([1, 2, 3], prompts)
+    out.append(lg)
+    for t in steps:
+        out.append(ctx.decode_step([1, 2, 3], t)[0])
+np.save({path!r}, np.stack(out[1:]))
+"""
+
+
+def _launch_run(tmp_path, name, env):
+    import os
+    import subprocess
+    import sys
+
+    root = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+    path = str(tmp_path / f"{name}.npy")
+    r = subprocess.run([sys.executable, "-c", _LAUNCH_RUN.format(root=root, path=path)], capture_output=True,
+                       text=True, env=dict(os.environ, **env), timeout=600)
+    assert r.returncode == 0, r.stderr[-2000:]
+    return np.load(path)
+
+
+def test_launch_paths_are_bitwise_identical(tlf, tmp_path):
+    """Graph replay with programmatic dependent launch, direct launches (TLF_NO_GRAPH=1) and plain
+    stream order (TLF_NO_PDL=1, read when the library loads) give identical decode logits."""
+    base = _launch_run(tmp_path, "base", {})
+    np.testing.assert_array_equal(_launch_run(tmp_path, "nograph", {"TLF_NO_GRAPH": "1"}), base)
+    np.testing.assert_array_equal(_launch_run(tmp_path, "nopdl", {"TLF_NO_PDL": "1"}), base)
+
+
 # ----------------------------------------------------------------------------
 # ablations: the same logits and loop counts as the method, different work
 # ----------------------------------------------------------------------------
