@@ -1103,12 +1103,18 @@ static int ensure_prefill_buffers(tlf_ctx* ctx) {
   return TLF_OK;
 }
 
-static void gemm_pf(tlf_ctx* ctx, const DeviceMat& W, const CUtensorMap* xmap, GemmArgs a, cudaStream_t st) {
+// rows: the chunk's token count (an upper bound on the rows of every loop)
+static void gemm_pf(tlf_ctx* ctx, const DeviceMat& W, const CUtensorMap* xmap, GemmArgs a, int rows,
+                    cudaStream_t st) {
   a.N = W.N;
   a.K = W.K;
   a.err = ctx->d_err;
   a.splits = 1;
-  a.red_window = 128;  // stage 128 of the 256 token columns at a time: two CTAs per SM
+  // Stage 128 of the 256 token columns at a time (2-stage ring): two CTAs share an SM, so one
+  // CTA's epilogue overlaps the other's main loop. Only worth it when the grid has more tiles
+  // than SMs; a smaller grid keeps one CTA per SM and the deeper ring.
+  const long long tiles = (long long)((W.N + 127) / 128) * ((rows + 255) / 256);
+  a.red_window = tiles > ctx->num_sms ? 128 : 0;
   a.max_rows = ctx->pf_C;
   a.tok_tiles = ctx->pf_C / 256;
   launch_gemm_tc(&W.map, xmap, 256, a, st);
@@ -1248,7 +1254,7 @@ static int prefill_batched(tlf_ctx* ctx, int n_seqs, const int* slot_of, const i
         a.row_slot = ctx->d_pf_row_slot + (size_t)r * C;
         a.row_cslot = ctx->d_pf_row_cslot + (size_t)r * C;
         a.row_pos = ctx->d_pf_row_pos + (size_t)r * C;
-        gemm_pf(ctx, ctx->wqkv[j], &ctx->pf_map_X, a, st);
+        gemm_pf(ctx, ctx->wqkv[j], &ctx->pf_map_X, a, T, st);
         launch_pf_attn(md, P, sp, r, j, ctx->d_pf_Q, ctx->d_pf_O, C / P.qblock + S + 1, st);
         a = GemmArgs{};
         a.n_dev = n_dev;
@@ -1257,7 +1263,7 @@ static int prefill_batched(tlf_ctx* ctx, int n_seqs, const int* slot_of, const i
         a.ldr = md.d;
         a.idx = idx_r;
         a.alpha = cond_args(ctx, ctx->d_pf_m, r, j, 0);
-        gemm_pf(ctx, ctx->wo[j], &ctx->pf_map_O, a, st);
+        gemm_pf(ctx, ctx->wo[j], &ctx->pf_map_O, a, T, st);
         launch_norm_rows(md.dtype, ctx->d_pf_H, md.d, idx_r, n_dev, 0, C, ctx->d_mlp_norm + (size_t)j * md.d, md.d,
                          md.eps, ctx->d_pf_X, md.d, st, cond_args(ctx, ctx->d_pf_m, r, j, 3));
         a = GemmArgs{};
@@ -1265,7 +1271,7 @@ static int prefill_batched(tlf_ctx* ctx, int n_seqs, const int* slot_of, const i
         a.epi = EPI_CL_SWIGLU;
         a.md = md;
         a.U = ctx->d_pf_U;
-        gemm_pf(ctx, ctx->wgu[j], &ctx->pf_map_X, a, st);
+        gemm_pf(ctx, ctx->wgu[j], &ctx->pf_map_X, a, T, st);
         a = GemmArgs{};
         a.n_dev = n_dev;
         a.epi = EPI_CL_RESID;
@@ -1273,7 +1279,7 @@ static int prefill_batched(tlf_ctx* ctx, int n_seqs, const int* slot_of, const i
         a.ldr = md.d;
         a.idx = idx_r;
         a.alpha = cond_args(ctx, ctx->d_pf_m, r, j, 1);
-        gemm_pf(ctx, ctx->wd[j], &ctx->pf_map_U, a, st);
+        gemm_pf(ctx, ctx->wd[j], &ctx->pf_map_U, a, T, st);
       }
     }
     if (last_logits && nend > 0) {
