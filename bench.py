@@ -280,31 +280,70 @@ def run_ours(args):
             torch.distributed.barrier()
         torch.cuda.synchronize()
 
+    # L2 between timed steps: a step whose working set (weights + the KV pages in use) is at least
+    # twice the L2 streams from HBM anyway; a smaller one gets the L2 flushed (a write larger than
+    # it) before every timed step, outside the timed intervals.
+    eb_w = 2 if m.dtype == "bf16" else 4
+    l2_bytes = int(getattr(torch.cuda.get_device_properties(local), "L2_cache_size", 0) or (128 << 20))
+    _, free_pages, total_pages = ctx.stats()
+    working_set = (m.n_layers * m.layer_params() + m.vocab * m.d_model) * eb_w + \
+        (total_pages - free_pages) * T.tlf_page_bytes(ctx.cfg)
+    flush_buf = torch.empty(2 * l2_bytes // 4, dtype=torch.int32, device="cuda") if working_set < 2 * l2_bytes \
+        else None
+    l2_note = ("L2 flushed before every timed step (a %d MB write outside the timed intervals; working set %d MB)"
+               % (2 * l2_bytes >> 20, working_set >> 20)) if flush_buf is not None else \
+        ("inputs larger than L2 (working set %d MB: KV cache and weights stream from HBM every step)"
+         % (working_set >> 20))
+
     # --- device-timed pass (logits stay on the device) ---
     for s in range(args.warmup):
         ctx.decode_step(ids, toks[s], forced=forced, logits=logits_dev, stream=stream)
     clocks = ClockSampler(local, os.path.join(ROOT, "gpurun_out" if os.path.isdir(os.path.join(ROOT, "gpurun_out"))
                                               else "_work", f"clocks_rank{rank}.csv"))
     barrier()
-    ev = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps + 1)]
-    ev[0].record(stream)
     loops_seen = []
-    for s in range(args.steps):
-        _, lp, _ = ctx.decode_step(ids, toks[args.warmup + s], forced=forced, logits=logits_dev, stream=stream)
-        ev[s + 1].record(stream)
-        loops_seen.append(lp)
-    barrier()
+    if flush_buf is None:
+        ev = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps + 1)]
+        ev[0].record(stream)
+        for s in range(args.steps):
+            _, lp, _ = ctx.decode_step(ids, toks[args.warmup + s], forced=forced, logits=logits_dev, stream=stream)
+            ev[s + 1].record(stream)
+            loops_seen.append(lp)
+        barrier()
+        step_ms = [ev[i].elapsed_time(ev[i + 1]) for i in range(args.steps)]
+        total_ms = ev[0].elapsed_time(ev[-1])
+    else:
+        st_ev = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps)]
+        en_ev = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps)]
+        for s in range(args.steps):
+            flush_buf.zero_()
+            st_ev[s].record(stream)
+            _, lp, _ = ctx.decode_step(ids, toks[args.warmup + s], forced=forced, logits=logits_dev, stream=stream)
+            en_ev[s].record(stream)
+            loops_seen.append(lp)
+        barrier()
+        step_ms = [st_ev[i].elapsed_time(en_ev[i]) for i in range(args.steps)]
+        total_ms = float(sum(step_ms))
     clk = clocks.stop()
-    step_ms = [ev[i].elapsed_time(ev[i + 1]) for i in range(args.steps)]
-    total_ms = ev[0].elapsed_time(ev[-1])
 
     # --- end-to-end pass: host tokens in, host logits out ---
     barrier()
-    t = time.perf_counter()
-    for s in range(args.steps):
-        ctx.decode_step(ids, toks[n_steps + s], forced=forced, logits=logits_host, stream=stream)
-    barrier()
-    e2e_ms = (time.perf_counter() - t) * 1e3
+    if flush_buf is None:
+        t = time.perf_counter()
+        for s in range(args.steps):
+            ctx.decode_step(ids, toks[n_steps + s], forced=forced, logits=logits_host, stream=stream)
+        barrier()
+        e2e_ms = (time.perf_counter() - t) * 1e3
+    else:
+        e2e_ms = 0.0
+        for s in range(args.steps):
+            flush_buf.zero_()
+            torch.cuda.synchronize()
+            t = time.perf_counter()
+            ctx.decode_step(ids, toks[n_steps + s], forced=forced, logits=logits_host, stream=stream)
+            torch.cuda.synchronize()
+            e2e_ms += (time.perf_counter() - t) * 1e3
+        barrier()
 
     # --- kernel-level pass: attention kernel time and algorithmic KV bytes ---
     ctx.set_profiling(True)
@@ -348,7 +387,7 @@ def run_ours(args):
             "data": "synthetic",
             "config": {"workload": DESCR[args.config], "name": args.config, "batch_per_gpu": B,
                        "context": int(wl.prompt_len[1]), "cache": how,
-                       "l2": "inputs larger than L2 (KV cache and weights stream from HBM every step)",
+                       "l2": l2_note,
                        "parallelism": f"replicas x{ws} (independent sequences per GPU)",
                        "ablation": args.ablation},
             "mean_loops": float(loops_seen.mean()),
