@@ -155,8 +155,6 @@ __device__ __forceinline__ void bulk_g2s(uint32_t dst, const void* src, uint32_t
       : "memory");
 }
 
-// 2-D tiled tensor copy global -> shared with a tensor map (coordinates in elements,
-// innermost first). The innermost coordinate times the element size is a multiple of 16.
 // L2 access policies for the cache_hint forms of the bulk copies: streamed data
 // that is read once per launch (KV pages, decode weight tiles) is marked for
 // early eviction so it does not displace the step's small, reused buffers.
@@ -181,7 +179,9 @@ __device__ __forceinline__ void bulk_g2s_hint(uint32_t dst, const void* src, uin
       : "memory");
 }
 
-// tma_load_2d with an L2 access policy.
+// 2-D tiled tensor copy global -> shared with a tensor map (coordinates in elements,
+// innermost first). The innermost coordinate times the element size is a multiple of 16.
+// This form carries an L2 access policy; tma_load_2d below has none.
 __device__ __forceinline__ void tma_load_2d_hint(uint32_t dst, const CUtensorMap* map, int32_t c0, int32_t c1,
                                                  uint32_t bar, uint64_t policy) {
   asm volatile(
@@ -470,9 +470,11 @@ struct GemmArgs {
   // offset max_rows, and the GEMM multiplies both (MMA N = 2 x tile, halves summed in the
   // epilogue), so the operand keeps about 16 significant bits instead of 8.
   int blo;                 // consumer: row offset of the token operand's lo plane (0: one plane)
-  int red_window;          // cluster epilogues with one split: token columns staged per pass (0: all)
   bf16* xn_lo;             // producer (split norm): lo plane of xn (NULL: none)
   void* U_lo;              // EPI_CL_SWIGLU: lo plane of U (NULL: none)
+  // One-split cluster epilogues (prefill) may stage their fp32 tile in windows of this many token
+  // columns, so the CTA needs less shared memory and two share an SM (0: the whole tile at once).
+  int red_window;
 };
 // Entries per row of the split-norm partial sums for model width d.
 inline int split_norm_ldss(int d) { return (((d + 127) / 128) + 3) / 4 * 4; }
