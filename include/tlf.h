@@ -171,10 +171,15 @@ int tlf_validate_config(const tlf_config* cfg, char* msg, size_t msg_len);
  * (sequence, loop) cache. Returns 0 for an invalid config. */
 int64_t tlf_page_bytes(const tlf_config* cfg);
 
-/* Create a context: validate cfg, copy the weights to the current CUDA
- * device, allocate the KV page pool and step workspaces. *out receives the
- * context (NULL on failure). On failure the message is available through
- * tlf_last_error(NULL) on the same thread.
+/* Create a context (Sec. 3.2-3.3): validate cfg, copy the weights of the
+ * shared J-layer block, the router and the tied embedding to the current CUDA
+ * device, and allocate the KV page pool that holds the recursion-wise caches
+ * of Sec. 3.3 (Eq. 8: one cache per loop i <= M, the user-set maximum depth
+ * of Sec. 3.2, and per layer j) plus the step workspaces. Weights are copied;
+ * the caller keeps ownership of w. *out receives the context (NULL on
+ * failure). On failure the message is available through tlf_last_error(NULL)
+ * on the same thread. Errors: INVALID_ARG (cfg), BAD_WEIGHTS (a required
+ * pointer is NULL), CUDA (no sm_103a device, allocation failure).
  *
  * Environment switches select equivalent comparison paths, each covered by
  * the GPU tests. The first two change only how kernels are launched, and the
@@ -191,7 +196,10 @@ int64_t tlf_page_bytes(const tlf_config* cfg);
  *                        here) */
 int tlf_create(const tlf_config* cfg, const tlf_weights* w, tlf_ctx** out);
 
-/* Free every device and host resource of the context. NULL is a no-op. */
+/* Free every device and host resource of the context: the weights, the
+ * page pool with every sequence's recursion-wise caches (Sec. 3.3, Eq. 8) and
+ * the workspaces. Live sequences end with it. NULL is a no-op. Synchronises
+ * the device before freeing, so no queued step reads freed memory. */
 void tlf_destroy(tlf_ctx* ctx);
 
 /* Message of the last failed call on ctx (or of the last failed tlf_create
@@ -234,7 +242,10 @@ int tlf_decode_step(tlf_ctx* ctx, int32_t batch, const uint64_t* seq_ids, const 
                     const int32_t* forced, float* logits, int32_t* loops, float* router_margin,
                     void* stream);
 
-/* End a sequence and return the pages of all M loop caches to the pool. */
+/* End a sequence: return the pages of its M recursion-wise caches (Sec. 3.3,
+ * Eq. 8: the loop-i caches of every layer j) to the pool and free its slot.
+ * The id may be reused by a later tlf_prefill or tlf_load_cache. Host-side
+ * only: queues no device work. Errors: UNKNOWN_SEQ. */
 int tlf_release(tlf_ctx* ctx, uint64_t seq_id);
 
 /* Create a sequence whose recursion-wise caches hold a given snapshot (a
@@ -305,7 +316,10 @@ int tlf_attn_decode(const tlf_attn_args* a, void* scratch, size_t scratch_bytes,
  * 4 MiB are rejected with TLF_ERR_INVALID_ARG and a message naming the
  * sizes; a C4-shaped call (16 rows, Hq 16 / Hkv 8, hd 128) needs under 1
  * MiB. The first call on a device looks up the array's device address (a
- * set-up step), so make that first call before any stream capture. Every
+ * set-up step), so make that first call before any stream capture. The
+ * address is remembered per device and per CUDA context: after the context
+ * is destroyed and re-created (cudaDeviceReset, for one) the next call looks
+ * it up again, so make that call, too, before any stream capture. Every
  * call on a device shares the array and it keeps the last call's contents:
  * calls whose kernels overlap on the GPU (different streams, or other host
  * threads) race and must not be issued; serialise them. Launches on

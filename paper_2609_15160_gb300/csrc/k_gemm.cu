@@ -14,9 +14,10 @@
 // - All four warps then read the accumulator with tcgen05.ld (warp w owns TMEM
 //   lanes 32w..32w+31 = output features) and run the epilogue. Split-K over
 //   gridDim.y keeps enough CTAs in flight to stream the weights at HBM speed.
-// Two-term operands (decode, token tiles <= 64): the token operand arrives as
-// bf16 hi and lo planes, loaded as one B tile of 2 x NT rows; the MMA runs with
-// N = 2 x NT and the epilogue adds the two accumulator halves.
+// Two-term operands (decode): the token operand arrives as bf16 hi and lo
+// planes, loaded as one B tile of 2 x NT rows; the MMA runs with N = 2 x NT
+// (two MMAs of N = 256 for a 256-token tile, whose halves fill TMEM) and the
+// epilogue adds the two accumulator halves.
 //
 // k_gemm_simt: CUDA-core tiled GEMM with the same epilogues, for float32
 // models (tcgen05 has no exact float32 mode) and as a second GPU path.
@@ -78,27 +79,32 @@ constexpr int tc_body_bytes(int nt, int stages, bool lo, int red_cols) {
   return tc_ring_bytes(nt, stages, lo) > tc_red_bytes(red_cols) ? tc_ring_bytes(nt, stages, lo)
                                                                 : tc_red_bytes(red_cols);
 }
-// TMEM columns of one CTA: the accumulator of 2 x NT columns (hi and lo halves) for
-// token tiles that may take a two-term operand, NT otherwise, at least 32.
-constexpr int tc_tmem_cols(int nt) {
-  return nt <= GEMM_LO_MAX_NT ? (2 * nt < 32 ? 32 : 2 * nt) : (nt < 32 ? 32 : nt);
+// TMEM columns of one CTA: the accumulator of 2 x NT columns (hi and lo halves) with a
+// two-term operand, NT otherwise, at least 32 (always a power of two).
+constexpr int tc_tmem_cols(int nt, bool lo) {
+  return lo ? (2 * nt < 32 ? 32 : 2 * nt) : (nt < 32 ? 32 : nt);
 }
 // tcgen05.alloc blocks until columns are free, so the CTAs that shared memory lets
 // share an SM must fit in its 512 TMEM columns (otherwise clusters waiting for
 // partners could wait on each other): launches request at least this much.
 constexpr int SM_SMEM = 232448;  // shared memory per SM available to CTAs (227 KB + 1 KB per CTA)
-constexpr int tc_min_smem(int nt) { return SM_SMEM / (512 / tc_tmem_cols(nt) + 1) - 1024 + 1; }
+constexpr int tc_min_smem(int nt, bool lo) { return SM_SMEM / (512 / tc_tmem_cols(nt, lo) + 1) - 1024 + 1; }
 constexpr int tc_smem_bytes(int nt, int stages, bool lo, int red_cols = 0) {
   const int raw = 1024 /*align slack*/ + tc_body_bytes(nt, stages, lo, red_cols > 0 ? red_cols : nt) +
                   256 /*barriers, tmem slot*/ +
                   nt * (16 + 4 + 16);
-  return raw > tc_min_smem(nt) ? raw : tc_min_smem(nt);
+  return raw > tc_min_smem(nt, lo) ? raw : tc_min_smem(nt, lo);
 }
-constexpr bool tmem_fits(int nt) {
-  return (SM_SMEM / (tc_smem_bytes(nt, 1, false) + 1024)) * tc_tmem_cols(nt) <= 512;
+// Deepest operand ring of a token tile: a 256-token two-term stage holds 80 KB, so two fit.
+constexpr int tc_max_stages(int nt, bool lo) { return (lo && nt >= 256) ? 2 : TC_STAGES; }
+constexpr bool tmem_fits(int nt, bool lo) {
+  return (SM_SMEM / (tc_smem_bytes(nt, 1, lo) + 1024)) * tc_tmem_cols(nt, lo) <= 512 &&
+         tc_smem_bytes(nt, tc_max_stages(nt, lo), lo) <= SM_SMEM - 1024;
 }
-static_assert(tmem_fits(16) && tmem_fits(32) && tmem_fits(64) && tmem_fits(128) && tmem_fits(256),
-              "co-resident CTAs would oversubscribe TMEM");
+static_assert(tmem_fits(16, false) && tmem_fits(32, false) && tmem_fits(64, false) && tmem_fits(128, false) &&
+                  tmem_fits(256, false) && tmem_fits(16, true) && tmem_fits(32, true) && tmem_fits(64, true) &&
+                  tmem_fits(128, true) && tmem_fits(256, true),
+              "co-resident CTAs would oversubscribe TMEM, or a ring does not fit in shared memory");
 
 // Second half of a cluster epilogue. Every CTA of the cluster has staged its
 // fp32 partial tile [NT columns][128 features] at `red`; this CTA sums the
@@ -361,8 +367,8 @@ template <int NT>
 __global__ void __launch_bounds__(128) k_gemm_tc(const __grid_constant__ CUtensorMap mapW,
                                                  const __grid_constant__ CUtensorMap mapX, GemmArgs a) {
   constexpr int A_BYTES = TC_BM * TC_BK * 2;
-  constexpr uint32_t TMEM_COLS = tc_tmem_cols(NT);
-  const bool lo = NT <= GEMM_LO_MAX_NT && a.blo > 0;  // two-term token operand
+  const bool lo = a.blo > 0;  // two-term token operand
+  const uint32_t TMEM_COLS = (uint32_t)tc_tmem_cols(NT, lo);
   const int B_BYTES = tc_b_bytes(NT, lo);
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
@@ -488,8 +494,12 @@ __global__ void __launch_bounds__(128) k_gemm_tc(const __grid_constant__ CUtenso
   if (nk > 0) {
     if (warp == 1 && lane == 0) {
       // MMA issuer
-      // a two-term operand: MMA N covers the hi rows (NT) and the lo rows (NT)
-      const uint32_t idesc = idesc_bf16_f32(TC_BM, lo ? 2 * NT : ncols);
+      // a two-term operand: MMA N covers the hi rows (NT) and the lo rows (NT); N is at most
+      // 256, so a 256-token tile multiplies its lo rows (32 KB further into the stage) in a
+      // second MMA into TMEM columns 256..511
+      constexpr bool SPLIT_LO = 2 * NT > 256;
+      const uint32_t idesc = idesc_bf16_f32(TC_BM, lo ? (SPLIT_LO ? NT : 2 * NT) : ncols);
+      constexpr uint64_t LO_DESC_OFF = (uint64_t)(NT * TC_BK * 2) >> 4;  // encoded start-address step
       for (int i = 0; i < nk; ++i) {
         const int st = i % NS;
         const uint32_t ph = (uint32_t)(i / NS) & 1u;
@@ -498,8 +508,11 @@ __global__ void __launch_bounds__(128) k_gemm_tc(const __grid_constant__ CUtenso
         const uint64_t da = smem_desc_sw128(smem_u32(sA + st * A_BYTES));
         const uint64_t db = smem_desc_sw128(smem_u32(sB + st * B_BYTES));
 #pragma unroll
-        for (int k = 0; k < TC_BK / 16; ++k)  // +32 bytes per K step of 16 bf16 (encoded >> 4)
-          tc_mma_f16(tmem, da + 2 * k, db + 2 * k, idesc, (i > 0 || k > 0) ? 1u : 0u);
+        for (int k = 0; k < TC_BK / 16; ++k) {  // +32 bytes per K step of 16 bf16 (encoded >> 4)
+          const uint32_t acc = (i > 0 || k > 0) ? 1u : 0u;
+          tc_mma_f16(tmem, da + 2 * k, db + 2 * k, idesc, acc);
+          if (SPLIT_LO && lo) tc_mma_f16(tmem + (uint32_t)NT, da + 2 * k, db + LO_DESC_OFF + 2 * k, idesc, acc);
+        }
         tc_commit(empty(st));
       }
       tc_commit(done);
@@ -584,10 +597,11 @@ __global__ void __launch_bounds__(128) k_gemm_tc(const __grid_constant__ CUtenso
   if (warp == 0) tmem_dealloc(tmem, TMEM_COLS);
 }
 
-int gemm_tc_stages(int K, int splits) {
+int gemm_tc_stages(int K, int splits, int nt, bool lo) {
   const int nkb = (K + TC_BK - 1) / TC_BK;
   const int per_cta = (nkb + splits - 1) / splits;
-  return per_cta < 1 ? 1 : (per_cta > TC_STAGES ? TC_STAGES : per_cta);
+  const int cap = tc_max_stages(nt, lo);
+  return per_cta < 1 ? 1 : (per_cta > cap ? cap : per_cta);
 }
 
 int gemm_tc_smem_bytes(int nt, int stages, bool lo) { return tc_smem_bytes(nt, stages, lo); }
@@ -597,12 +611,12 @@ template <int NT>
 static void launch_tc_nt(const CUtensorMap* mapW, const CUtensorMap* mapX, GemmArgs a, cudaStream_t st) {
   static bool attr_set = false;
   if (!attr_set) {
-    cudaFuncSetAttribute(k_gemm_tc<NT>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                         tc_smem_bytes(NT, TC_STAGES, NT <= GEMM_LO_MAX_NT));
+    const int one = tc_smem_bytes(NT, tc_max_stages(NT, false), false);
+    const int two = tc_smem_bytes(NT, tc_max_stages(NT, true), true);
+    cudaFuncSetAttribute(k_gemm_tc<NT>, cudaFuncAttributeMaxDynamicSharedMemorySize, one > two ? one : two);
     attr_set = true;
   }
-  a.stages = gemm_tc_stages(a.K, a.splits);
-  if (NT > GEMM_LO_MAX_NT) a.blo = 0;
+  a.stages = gemm_tc_stages(a.K, a.splits, NT, a.blo > 0);
   int red_cols = NT;
   if (a.red_window > 0 && a.splits == 1 && a.red_window < NT) {
     // windowed one-split epilogue: with a 2-stage ring two CTAs share an SM, so one CTA's

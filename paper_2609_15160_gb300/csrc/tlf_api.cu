@@ -481,10 +481,10 @@ static int create_impl(tlf_ctx* ctx, const tlf_weights* w) {
   if ((rc = dev_alloc(ctx, &ctx->d_margin, (size_t)B * 4, "margin"))) return rc;
   if ((rc = dev_alloc(ctx, &ctx->d_H, (size_t)B * d * 4, "H"))) return rc;
   {
-    // two-term operands (hi + lo planes) where the token tile allows it; TLF_NO_OPERAND_LO=1
-    // keeps one bf16 plane (comparison runs)
+    // two-term operands (hi + lo planes) for every decode GEMM of the tcgen05 path;
+    // TLF_NO_OPERAND_LO=1 keeps one bf16 plane (comparison runs)
     const char* e = getenv("TLF_NO_OPERAND_LO");
-    ctx->operand_lo = ctx->use_tc && ctx->nt_max <= GEMM_LO_MAX_NT && !(e && e[0] == '1');
+    ctx->operand_lo = ctx->use_tc && !(e && e[0] == '1');
   }
   const int planes = ctx->operand_lo ? 2 : 1;
   if ((rc = dev_alloc(ctx, &ctx->d_X, (size_t)planes * B * d * eb, "X"))) return rc;
@@ -509,7 +509,8 @@ static int create_impl(tlf_ctx* ctx, const tlf_weights* w) {
     auto pick = [&](int tiles, int K) {
       const int nkb = (K + 63) / 64;
       for (int S = std::min(8, nkb); S > 1; --S) {
-        const int bytes = gemm_tc_smem_bytes(ctx->nt_max, gemm_tc_stages(K, S), ctx->operand_lo);
+        const int bytes =
+            gemm_tc_smem_bytes(ctx->nt_max, gemm_tc_stages(K, S, ctx->nt_max, ctx->operand_lo), ctx->operand_lo);
         const int per_sm = std::min(16, 232448 / (bytes + 1024));
         if (10LL * tiles * S <= 9LL * per_sm * ctx->num_sms) return S;
       }

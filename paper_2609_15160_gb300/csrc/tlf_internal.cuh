@@ -465,7 +465,7 @@ struct GemmArgs {
   const float* ss_in;      // consumer: [max_rows][ldss] (NULL: operand already normalised)
   int ldss;
   float norm_eps;
-  // Two-term bf16 operand (tcgen05 decode path, token tiles <= 64). An activation v is
+  // Two-term bf16 operand (tcgen05 decode path). An activation v is
   // stored as hi = bf16(v) and lo = bf16(v - hi) in two planes of one buffer, lo at row
   // offset max_rows, and the GEMM multiplies both (MMA N = 2 x tile, halves summed in the
   // epilogue), so the operand keeps about 16 significant bits instead of 8.
@@ -503,12 +503,11 @@ int build_cond_table(const ModelDims& md, const float* t_w1, const float* t_b1, 
 void launch_gemm_simt(int dtype, const void* W, const void* X, int ldx, const GemmArgs& a, cudaStream_t st);
 void launch_gemm_tc(const CUtensorMap* mapW, const CUtensorMap* mapX, int nt_max, const GemmArgs& a,
                     cudaStream_t st);
-// operand-ring depth of a tcgen05 GEMM whose CTAs each reduce ceil(ceil(K/64)/splits) k-tiles,
-// and the dynamic shared memory one CTA of token tile nt then needs
-int gemm_tc_stages(int K, int splits);
+// operand-ring depth of a tcgen05 GEMM whose CTAs each reduce ceil(ceil(K/64)/splits) k-tiles
+// with token tile nt (and a two-term operand when lo), and the dynamic shared memory one CTA
+// then needs
+int gemm_tc_stages(int K, int splits, int nt, bool lo);
 int gemm_tc_smem_bytes(int nt, int stages, bool lo = false);
-// largest token tile whose GEMMs take a two-term (hi + lo) operand
-constexpr int GEMM_LO_MAX_NT = 64;
 
 void launch_rope_table(const ModelDims& md, const double* inv_freq, float2* table, cudaStream_t st);
 void launch_rope_append(const ModelDims& md, const StepDev& s, int r, int j, const float* part, int splits,

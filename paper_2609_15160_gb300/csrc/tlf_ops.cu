@@ -6,6 +6,8 @@
 // lengths, the plan kernel cuts every (row, kv head) key range into chunks,
 // k_attn_decode streams the pages and k_attn_combine merges the chunk
 // partials. The scratch holds the plan and the partials.
+#include <atomic>
+
 #include "tlf.h"
 #include "tlf_internal.cuh"
 
@@ -64,17 +66,23 @@ const char* attn_op_validate(const tlf_attn_args* a) {
   if (a->n_layers < 1 || a->layer < 0 || a->layer >= a->n_layers) return "layer out of range";
   if (a->page_size != 64) return "page_size must be 64";
   if (a->max_pages < 1 || a->n_pages < 1 || a->n_pages > 0x7fffffff) return "bad page counts";
+  if (a->max_pages > 0x7fffffff / a->page_size) return "max_pages * page_size exceeds the int32 key range";
   if (!a->q || !a->pool || !a->page_table || !a->lens || !a->out) return "a device pointer is NULL";
   return nullptr;
 }
 
 int current_num_sms() {
-  static int cache[64] = {0};
+  // one entry per device ordinal, filled on first use; concurrent first uses store the same value
+  static std::atomic<int> cache[64];
   int dev = 0;
   if (cudaGetDevice(&dev) != cudaSuccess) return 0;
   if (dev < 0 || dev >= 64) return 0;
-  if (!cache[dev]) cudaDeviceGetAttribute(&cache[dev], cudaDevAttrMultiProcessorCount, dev);
-  return cache[dev];
+  int n = cache[dev].load(std::memory_order_relaxed);
+  if (!n) {
+    if (cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess) return 0;
+    cache[dev].store(n, std::memory_order_relaxed);
+  }
+  return n;
 }
 
 cudaError_t attn_op_run(const tlf_attn_args* a, uint8_t* scratch, const AttnOpLayout& L, cudaStream_t st) {

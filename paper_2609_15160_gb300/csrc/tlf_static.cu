@@ -5,7 +5,14 @@
 // split-K partials) is a fixed array in the library's device image instead
 // of a caller buffer. Host code cannot use the array's name as a device
 // address, so the first call on each device looks the address up with
-// cudaGetSymbolAddress while that device is current and remembers it.
+// cudaGetSymbolAddress while that device is current and remembers it, keyed
+// by the device and by the id of its current CUDA context: a context that is
+// torn down and re-created (cudaDeviceReset, for one) loads the module again,
+// possibly elsewhere, and gets a new id, so the next call looks again instead
+// of handing the kernels a stale address.
+#include <cudaTypedefs.h>
+
+#include <atomic>
 #include <cstdio>
 #include <mutex>
 
@@ -19,24 +26,58 @@ static __device__ __align__(256) uint8_t g_static_scratch[kStaticScratchBytes];
 namespace {
 std::mutex g_scratch_mu;
 constexpr int kMaxDevices = 64;
-void* g_scratch_addr[kMaxDevices] = {};
+struct ScratchEntry {
+  unsigned long long ctx_id = 0;  // CUDA context the address belongs to
+  void* addr = nullptr;
+};
+ScratchEntry g_scratch[kMaxDevices];
 
-// Device address of g_static_scratch on the current device (looked up once per device).
+// Id of the calling thread's current CUDA context (unique for the life of the process);
+// false when no context is current yet or the driver entry points are unavailable.
+bool current_context_id(unsigned long long* id) {
+  static std::atomic<PFN_cuCtxGetCurrent_v4000> get_current{nullptr};
+  static std::atomic<PFN_cuCtxGetId_v12000> get_id{nullptr};
+  if (!get_current.load() || !get_id.load()) {
+    void* p = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuCtxGetCurrent", &p, 4000, cudaEnableDefault, &q) != cudaSuccess ||
+        q != cudaDriverEntryPointSuccess || !p)
+      return false;
+    get_current.store(reinterpret_cast<PFN_cuCtxGetCurrent_v4000>(p));
+    p = nullptr;
+    if (cudaGetDriverEntryPointByVersion("cuCtxGetId", &p, 12000, cudaEnableDefault, &q) != cudaSuccess ||
+        q != cudaDriverEntryPointSuccess || !p)
+      return false;
+    get_id.store(reinterpret_cast<PFN_cuCtxGetId_v12000>(p));
+  }
+  CUcontext c = nullptr;
+  if (get_current.load()(&c) != CUDA_SUCCESS || !c) return false;
+  return get_id.load()(c, id) == CUDA_SUCCESS;
+}
+
+// Device address of g_static_scratch in the current device's current context (looked up
+// once per device and context).
 int static_scratch_address(void** out) {
   int dev = -1;
   cudaError_t e = cudaGetDevice(&dev);
   if (e != cudaSuccess) return tlf::set_thread_error(TLF_ERR_CUDA, cudaGetErrorString(e));
   if (dev < 0 || dev >= kMaxDevices) return tlf::set_thread_error(TLF_ERR_CUDA, "device ordinal out of range");
   std::lock_guard<std::mutex> lock(g_scratch_mu);
-  if (!g_scratch_addr[dev]) {
+  ScratchEntry& ent = g_scratch[dev];
+  unsigned long long id = 0;
+  const bool have_id = current_context_id(&id);
+  if (!have_id || !ent.addr || ent.ctx_id != id) {
     void* p = nullptr;
-    e = cudaGetSymbolAddress(&p, g_static_scratch);
+    e = cudaGetSymbolAddress(&p, g_static_scratch);  // makes the runtime's context current if none was
     if (e != cudaSuccess || !p)
       return tlf::set_thread_error(TLF_ERR_CUDA, e != cudaSuccess ? cudaGetErrorString(e)
                                                                   : "cudaGetSymbolAddress returned NULL");
-    g_scratch_addr[dev] = p;
+    if (!current_context_id(&id))
+      return tlf::set_thread_error(TLF_ERR_CUDA, "no current CUDA context after the symbol lookup");
+    ent.ctx_id = id;
+    ent.addr = p;
   }
-  *out = g_scratch_addr[dev];
+  *out = ent.addr;
   return TLF_OK;
 }
 }  // namespace

@@ -60,16 +60,22 @@ def check_active_sets(ctx, loops, M, ablation="none"):
         np.testing.assert_array_equal(sets[r], want)
 
 
-def cache_tol(model):
+def cache_tol(model, prefilled=True):
     """Tolerance of a stored K/V entry row (max abs diff / row max).
 
     An entry of loop i is an intermediate result: it carries the error that
     bf16 activations accumulate over up to M x J layer applications (the same
     error the logits carry) plus one bf16 storage rounding (<= 2^-9 of the
-    entry), and a K/V row is normalised by the max of far fewer values than a
-    logits row. So the logits bound is widened by half for bf16 models.
+    entry), normalised by the max of a row of Hkv x hd values.
+    * Entries written by decode steps (two-term GEMM operands): measured worst
+      3.9e-3 over the C3/C4/C5 snapshot runs; bar 1e-2.
+    * Caches that also hold prefilled entries (the prefill GEMMs take one bf16
+      plane per operand): measured worst 1.78e-2 on the C4 model (12 layer
+      applications, d 2048); bar 2e-2.
     """
-    return 1e-4 if model.dtype == "f32" else 3e-2
+    if model.dtype == "f32":
+        return 1e-4
+    return 2e-2 if prefilled else 1e-2
 
 
 def check_cache(ctx, seq_id, oseq, model, tol=None, masked_slots=False):
@@ -80,6 +86,7 @@ def check_cache(ctx, seq_id, oseq, model, tol=None, masked_slots=False):
     the K/V of the unmasked slots are compared.
     """
     tol = cache_tol(model) if tol is None else tol
+    worst = 0.0
     for i in range(model.max_loops):
         for j in range(model.n_layers):
             gp, gk, gv = ctx.read_cache(seq_id, i + 1, j)
@@ -97,7 +104,10 @@ def check_cache(ctx, seq_id, oseq, model, tol=None, masked_slots=False):
                 g2, o2 = g.reshape(len(op), -1).astype(np.float64), o.reshape(len(op), -1).astype(np.float64)
                 row = np.max(np.abs(g2 - o2), axis=1) / np.max(np.abs(o2), axis=1)
                 bad = int(np.argmax(row))
+                worst = max(worst, float(row[bad]))
                 assert row[bad] < tol, (f"cache {name} loop {i + 1} layer {j}: entry {bad}/{len(op)} "
                                         f"(pos {op[bad]}) rel err {row[bad]:.3e}; rows over tol: "
                                         f"{np.nonzero(row >= tol)[0][:10].tolist()} gpu {g2[bad, :4]} "
                                         f"oracle {o2[bad, :4]}")
+    print(f"cache of sequence {seq_id}: worst K/V row rel err {worst:.3e} (bar {tol:.0e})")
+    return worst
