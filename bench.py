@@ -25,6 +25,7 @@ import os
 import statistics
 import subprocess
 import sys
+import tempfile
 import time
 
 import numpy as np
@@ -67,23 +68,26 @@ def _attn_traffic(alg_bytes_per_launch: float):
 
 
 class ClockSampler:
-    """nvidia-smi clock / throttle samples during the timed region."""
+    """nvidia-smi clock / throttle samples (every 20 ms) while a workload runs, in a temporary file."""
 
     Q = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
          "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
          "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
 
-    def __init__(self, gpu: int, path: str):
-        self.path, self.proc = path, None
+    def __init__(self, gpu: int):
+        self.proc = None
+        fd, self.path = tempfile.mkstemp(prefix="tlf_clocks_", suffix=".csv")
+        self.f = os.fdopen(fd, "w")
         try:
-            self.f = open(path, "w")
             self.proc = subprocess.Popen(["nvidia-smi", f"--id={gpu}", f"--query-gpu={self.Q}", "--format=csv",
-                                          "-lms", "200"], stdout=self.f, stderr=subprocess.DEVNULL)
+                                          "-lms", "20"], stdout=self.f, stderr=subprocess.DEVNULL)
         except (OSError, FileNotFoundError):
             self.proc = None
 
     def stop(self):
         if self.proc is None:
+            self.f.close()
+            os.unlink(self.path)
             return None
         self.proc.terminate()
         try:
@@ -93,7 +97,10 @@ class ClockSampler:
         self.f.close()
         sm, mx, reasons = [], [], set()
         names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
-        for line in open(self.path).read().splitlines()[1:]:
+        with open(self.path) as f:
+            lines = f.read().splitlines()[1:]
+        os.unlink(self.path)
+        for line in lines:
             parts = [x.strip() for x in line.split(",")]
             if len(parts) < 9:
                 continue
@@ -108,7 +115,7 @@ class ClockSampler:
         if not sm:
             return None
         return {"sm_mhz": statistics.median(sm), "sm_max_mhz": max(mx), "reasons": sorted(reasons),
-                "samples": len(sm)}
+                "samples": len(sm), "window": "warm-up, device-timed and end-to-end passes, 20 ms poll"}
 
 
 def _dist():
@@ -197,9 +204,19 @@ def run_reference(args):
     print(json.dumps(line))
 
 
+_WEIGHTS = {}
+
+
+def model_weights(m):
+    """Seeded weights of a model, generated once per model in this process (C3 and C5 share them)."""
+    if m not in _WEIGHTS:
+        _WEIGHTS[m] = synth.make_weights(m)
+    return _WEIGHTS[m]
+
+
 def setup_workload(T, wl, rank: int, gemm_impl="auto", prefill="auto", extra_tokens: int = 0, ablation="none"):
     m = wl.model
-    w = synth.make_weights(m)
+    w = model_weights(m)
     B = wl.batch
     prompts = synth.make_prompts(wl)
     lengths = [len(p) for p in prompts]
@@ -248,28 +265,36 @@ def setup_workload(T, wl, rank: int, gemm_impl="auto", prefill="auto", extra_tok
     return ctx, ids, how
 
 
-def run_ours(args):
+def gemm_operands(m, gemm_impl="auto"):
+    """Which operand path the decode GEMMs of this model take."""
+    if m.dtype != "bf16" or gemm_impl != "auto":
+        return "CUDA-core GEMM, operands in the model dtype"
+    if os.environ.get("TLF_NO_OPERAND_LO") == "1":
+        return "tcgen05, one bf16 plane per activation operand"
+    return "tcgen05, two-term bf16 activation operands (hi + lo planes)"
+
+
+NEAR_TIE = 1e-3
+
+
+def measure(T, wl, args, rank: int, ws: int, local: int, steps: int, warmup: int, breakdown: bool = True):
+    """Prefill the workload through the library, then time decode steps three ways.
+
+    device-timed: CUDA events on the launching stream, logits left on the device;
+    end to end: the public call with host token ids in and host logits out (copies timed);
+    profiled: per-kernel events, for the attention roofline and the kernel breakdown.
+    Returns the raw figures of this rank.
+    """
     import torch
 
-    from paper_2609_15160_gb300 import tlf as T
-
-    ws, rank, local = _dist()
-    torch.cuda.set_device(local)
-    if ws > 1:
-        import torch.distributed as dist
-        dist.init_process_group("nccl")
-    T.load_library()
-    wl = synth.get_config(args.config)
-    if args.decode_batch:
-        wl = wl.with_batch(args.decode_batch)
     m = wl.model
     B = wl.batch
     t0 = time.time()
-    ctx, ids, how = setup_workload(T, wl, rank, prefill=args.prefill,
-                                   extra_tokens=3 * (args.warmup + args.steps), ablation=args.ablation)
+    ctx, ids, how = setup_workload(T, wl, rank, prefill=args.prefill, extra_tokens=3 * (warmup + steps),
+                                   ablation=args.ablation)
     setup_s = time.time() - t0
     stream = torch.cuda.current_stream()
-    n_steps = args.warmup + args.steps
+    n_steps = warmup + steps
     toks = synth.make_decode_tokens(wl, steps=3 * n_steps + 2, batch=B)
     forced = None if wl.forced_loops is None else np.full(B, wl.forced_loops, np.int32)
     logits_dev = torch.empty((B, m.vocab), dtype=torch.float32, device="cuda")
@@ -296,47 +321,47 @@ def run_ours(args):
          % (working_set >> 20))
 
     # --- device-timed pass (logits stay on the device) ---
-    for s in range(args.warmup):
+    clocks = ClockSampler(local)
+    for s in range(warmup):
         ctx.decode_step(ids, toks[s], forced=forced, logits=logits_dev, stream=stream)
-    clocks = ClockSampler(local, os.path.join(ROOT, "gpurun_out" if os.path.isdir(os.path.join(ROOT, "gpurun_out"))
-                                              else "_work", f"clocks_rank{rank}.csv"))
     barrier()
-    loops_seen = []
+    loops_seen, margins = [], []
     if flush_buf is None:
-        ev = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps + 1)]
+        ev = [torch.cuda.Event(enable_timing=True) for _ in range(steps + 1)]
         ev[0].record(stream)
-        for s in range(args.steps):
-            _, lp, _ = ctx.decode_step(ids, toks[args.warmup + s], forced=forced, logits=logits_dev, stream=stream)
+        for s in range(steps):
+            _, lp, mg = ctx.decode_step(ids, toks[warmup + s], forced=forced, logits=logits_dev, stream=stream)
             ev[s + 1].record(stream)
             loops_seen.append(lp)
+            margins.append(mg)
         barrier()
-        step_ms = [ev[i].elapsed_time(ev[i + 1]) for i in range(args.steps)]
+        step_ms = [ev[i].elapsed_time(ev[i + 1]) for i in range(steps)]
         total_ms = ev[0].elapsed_time(ev[-1])
     else:
-        st_ev = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps)]
-        en_ev = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps)]
-        for s in range(args.steps):
+        st_ev = [torch.cuda.Event(enable_timing=True) for _ in range(steps)]
+        en_ev = [torch.cuda.Event(enable_timing=True) for _ in range(steps)]
+        for s in range(steps):
             flush_buf.zero_()
             st_ev[s].record(stream)
-            _, lp, _ = ctx.decode_step(ids, toks[args.warmup + s], forced=forced, logits=logits_dev, stream=stream)
+            _, lp, mg = ctx.decode_step(ids, toks[warmup + s], forced=forced, logits=logits_dev, stream=stream)
             en_ev[s].record(stream)
             loops_seen.append(lp)
+            margins.append(mg)
         barrier()
-        step_ms = [st_ev[i].elapsed_time(en_ev[i]) for i in range(args.steps)]
+        step_ms = [st_ev[i].elapsed_time(en_ev[i]) for i in range(steps)]
         total_ms = float(sum(step_ms))
-    clk = clocks.stop()
 
     # --- end-to-end pass: host tokens in, host logits out ---
     barrier()
     if flush_buf is None:
         t = time.perf_counter()
-        for s in range(args.steps):
+        for s in range(steps):
             ctx.decode_step(ids, toks[n_steps + s], forced=forced, logits=logits_host, stream=stream)
         barrier()
         e2e_ms = (time.perf_counter() - t) * 1e3
     else:
         e2e_ms = 0.0
-        for s in range(args.steps):
+        for s in range(steps):
             flush_buf.zero_()
             torch.cuda.synchronize()
             t = time.perf_counter()
@@ -344,81 +369,145 @@ def run_ours(args):
             torch.cuda.synchronize()
             e2e_ms += (time.perf_counter() - t) * 1e3
         barrier()
+    clk = clocks.stop()
 
     # --- kernel-level pass: attention kernel time and algorithmic KV bytes ---
     ctx.set_profiling(True)
     att_ms, att_bytes, launches, att_launches = 0.0, 0.0, 0, 0
-    breakdown = {}
-    for s in range(args.steps):
-        _, lp, _ = ctx.decode_step(ids, toks[2 * n_steps + s], forced=forced, logits=logits_dev, stream=stream)
+    kernel_ms = {}
+    for s in range(steps):
+        ctx.decode_step(ids, toks[2 * n_steps + s], forced=forced, logits=logits_dev, stream=stream)
         ms, by, nl = ctx.last_step_profile()
         att_ms += ms
         att_bytes += by
         launches += nl
         att_launches += m.n_layers * m.max_loops
-        for kname, kms in ctx.last_step_kernel_times().items():
-            breakdown[kname] = breakdown.get(kname, 0.0) + kms / args.steps
+        if breakdown:
+            for kname, kms in ctx.last_step_kernel_times().items():
+                kernel_ms[kname] = kernel_ms.get(kname, 0.0) + kms / steps
     ctx.set_profiling(False)
 
-    total_ms, e2e_ms = max_over_ranks([total_ms, e2e_ms], device="cuda")
     # algorithmic HBM bytes of the timed steps: the weights of every loop that had an active
     # token (read once per loop), the LM head, and the K/V every active token reads and writes
     eb = 2 if m.dtype == "bf16" else 4
     w_loop = m.n_layers * m.layer_params() * eb
     kv_entry = m.n_layers * 2 * m.n_kv_heads * m.head_dim * eb
-    step_bytes = []
-    for lp in loops_seen:
-        loops_run = int(lp.max())
-        step_bytes.append(loops_run * w_loop + m.vocab * m.d_model * eb + int(lp.sum()) * kv_entry)
-    kv_read_per_step = att_bytes / args.steps
-    alg_bytes = float(np.mean(step_bytes)) + kv_read_per_step
-    loops_seen = np.concatenate(loops_seen)
+    step_bytes = [int(lp.max()) * w_loop + m.vocab * m.d_model * eb + int(lp.sum()) * kv_entry for lp in loops_seen]
+    alg_bytes = float(np.mean(step_bytes)) + att_bytes / steps
+    r = dict(total_ms=total_ms, e2e_ms=e2e_ms, step_ms=step_ms, att_ms=att_ms, att_bytes=att_bytes,
+             launches=launches, att_launches=att_launches, kernel_ms=kernel_ms, alg_bytes=alg_bytes,
+             loops=np.concatenate(loops_seen), margins=np.concatenate(margins), how=how, l2_note=l2_note,
+             setup_s=setup_s, clocks=clk,
+             prefill=({"tokens": ctx.prefill_tokens, "seconds": ctx.prefill_seconds,
+                       "tokens_per_s": ctx.prefill_tokens / ctx.prefill_seconds}
+                      if hasattr(ctx, "prefill_seconds") else None))
+    ctx.close()
+    return r
+
+
+def summarize(wl, r, steps: int, ws: int, total_ms: float, e2e_ms: float, peak: float, peak_kind: str):
+    """Per-workload figures of the JSON line (rank 0, times already maxed over ranks)."""
+    m = wl.model
+    B = wl.batch
+    att_gbs = r["att_bytes"] / (r["att_ms"] * 1e-3) / 1e9 if r["att_ms"] > 0 else None
+    near = int(np.sum(np.abs(r["margins"]) <= NEAR_TIE)) if wl.forced_loops is None else 0
+    return {
+        "tokens_per_s": job_tokens_per_s(ws, B, steps, total_ms),
+        "ms_per_step": total_ms / steps,
+        "p50_step_ms": float(np.percentile(r["step_ms"], 50)),
+        "p90_step_ms": float(np.percentile(r["step_ms"], 90)),
+        "e2e_tokens_per_s": job_tokens_per_s(ws, B, steps, e2e_ms),
+        "step_roofline_frac": (r["alg_bytes"] / (peak * 1e9) * 1e3) / (total_ms / steps),
+        "step_floor_ms": r["alg_bytes"] / (peak * 1e9) * 1e3,
+        "attention_gbs": att_gbs,
+        "attention_frac": (att_gbs / peak) if att_gbs else None,
+        "mean_loops": float(r["loops"].mean()),
+        "depth_histogram": np.bincount(r["loops"], minlength=m.max_loops + 1)[1:].tolist(),
+        "near_tie_tokens": near,
+        "near_tie_rule": ("router margin <= 1e-3 among the timed tokens" if wl.forced_loops is None
+                          else "every token forced to %d loops: no router decision" % wl.forced_loops),
+        "gpu_launches": int(r["launches"]),
+    }
+
+
+# The five workloads beside the headline one, each timed in the same run (at one GPU).
+SUB_CONFIGS = ("c1", "c2", "c3", "c5", "c5f")
+
+
+def run_ours(args):
+    import torch
+
+    from paper_2609_15160_gb300 import tlf as T
+
+    ws, rank, local = _dist()
+    torch.cuda.set_device(local)
+    if ws > 1:
+        import torch.distributed as dist
+        dist.init_process_group("nccl")
+    T.load_library()
+    wl = synth.get_config(args.config)
+    if args.decode_batch:
+        wl = wl.with_batch(args.decode_batch)
+    m = wl.model
+    B = wl.batch
+    r = measure(T, wl, args, rank, ws, local, args.steps, args.warmup)
+    total_ms, e2e_ms = max_over_ranks([r["total_ms"], r["e2e_ms"]], device="cuda")
+    peak, peak_kind = _measured_peaks()
+    configs = {}
+    if ws == 1 and not args.no_configs:
+        for name in SUB_CONFIGS:
+            if name == args.config:
+                continue
+            swl = synth.get_config(name)
+            sr = measure(T, swl, args, rank, ws, local, args.steps, args.warmup, breakdown=False)
+            configs[name] = {"workload": DESCR[name], "batch": swl.batch, "cache": sr["how"], "l2": sr["l2_note"],
+                             "gemm_operands": gemm_operands(swl.model),
+                             **summarize(swl, sr, args.steps, ws, sr["total_ms"], sr["e2e_ms"], peak, peak_kind),
+                             "clocks": sr["clocks"]}
     if rank == 0:
-        peak, peak_kind = _measured_peaks()
-        att_gbs = att_bytes / (att_ms * 1e-3) / 1e9 if att_ms > 0 else None
-        value = job_tokens_per_s(ws, B, args.steps, total_ms)
+        s = summarize(wl, r, args.steps, ws, total_ms, e2e_ms, peak, peak_kind)
+        att_gbs = s["attention_gbs"]
         h2d = B * 12
         d2h = B * m.vocab * 4 + B * 8
         line = {
-            "metric": "decode_tokens_per_s", "value": value, "unit": "tokens/s", "n_gpus": ws,
-            "steps": args.steps, "warmup": args.warmup, "ms_per_step": total_ms / args.steps,
-            "p50_step_ms": float(np.percentile(step_ms, 50)), "p90_step_ms": float(np.percentile(step_ms, 90)),
+            "metric": "decode_tokens_per_s", "value": s["tokens_per_s"], "unit": "tokens/s", "n_gpus": ws,
+            "steps": args.steps, "warmup": args.warmup, "ms_per_step": s["ms_per_step"],
+            "p50_step_ms": s["p50_step_ms"], "p90_step_ms": s["p90_step_ms"],
             "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": m.dtype,
             "data": "synthetic",
             "config": {"workload": DESCR[args.config], "name": args.config, "batch_per_gpu": B,
-                       "context": int(wl.prompt_len[1]), "cache": how,
-                       "l2": l2_note,
+                       "context": int(wl.prompt_len[1]), "cache": r["how"],
+                       "l2": r["l2_note"],
                        "parallelism": f"replicas x{ws} (independent sequences per GPU)",
-                       "ablation": args.ablation},
-            "mean_loops": float(loops_seen.mean()),
-            "step_roofline": {"bound": "hbm", "algorithmic_bytes_per_step": alg_bytes,
-                              "floor_ms": alg_bytes / (peak * 1e9) * 1e3,
-                              "frac": (alg_bytes / (peak * 1e9) * 1e3) / (total_ms / args.steps),
+                       "ablation": args.ablation, "gemm_operands": gemm_operands(m)},
+            "mean_loops": s["mean_loops"],
+            "near_tie_tokens": s["near_tie_tokens"],
+            "step_roofline": {"bound": "hbm", "algorithmic_bytes_per_step": r["alg_bytes"],
+                              "floor_ms": s["step_floor_ms"], "frac": s["step_roofline_frac"],
                               "peak_gbs": peak, "peak_kind": peak_kind},
             "attention_gbs": att_gbs,
             "roofline": {"bound": "hbm", "kernel": "k_attn_decode (recursion-wise split-K attention)",
                          "achieved": att_gbs, "peak": peak, "unit": "GB/s",
                          "frac": (att_gbs / peak) if att_gbs else None, "peak_kind": peak_kind,
-                         "traffic": _attn_traffic(att_bytes / max(1, att_launches)),
+                         "traffic": _attn_traffic(r["att_bytes"] / max(1, r["att_launches"])),
                          "traffic_source": "ncu dram bytes / algorithmic bytes of one captured launch "
                                            "(profiles/traffic.json) x this launch's algorithmic bytes",
-                         "algorithmic_bytes_per_launch": att_bytes / max(1, att_launches),
-                         "avg_launch_ms": att_ms / max(1, att_launches)},
-            "e2e": {"value": job_tokens_per_s(ws, B, args.steps, e2e_ms), "unit": "tokens/s",
+                         "algorithmic_bytes_per_launch": r["att_bytes"] / max(1, r["att_launches"]),
+                         "avg_launch_ms": r["att_ms"] / max(1, r["att_launches"])},
+            "e2e": {"value": s["e2e_tokens_per_s"], "unit": "tokens/s",
                     "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h},
-            "gpu_launches": int(launches),
-            "kernel_ms_per_step_profiled": {k: round(v, 4) for k, v in breakdown.items()},
-            "setup_s": setup_s,
-            "prefill": ({"tokens": ctx.prefill_tokens, "seconds": ctx.prefill_seconds,
-                         "tokens_per_s": ctx.prefill_tokens / ctx.prefill_seconds}
-                        if hasattr(ctx, "prefill_seconds") else None),
+            "gpu_launches": s["gpu_launches"],
+            "kernel_ms_per_step_profiled": {k: round(v, 4) for k, v in r["kernel_ms"].items()},
+            "setup_s": r["setup_s"],
+            "prefill": r["prefill"],
         }
-        if clk:
-            line["clocks"] = clk
+        if r["clocks"]:
+            line["clocks"] = r["clocks"]
+        if configs:
+            line["configs"] = configs
         if not args.no_cpu_baseline and ws == 1:
             line["cpu_baseline"] = cpu_baseline(args.config)
         print(json.dumps(line))
-    ctx.close()
     if ws > 1:
         torch.distributed.destroy_process_group()
 
@@ -605,6 +694,9 @@ def main():
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--prefill", default="auto", choices=["auto", "snapshot", "real"])
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-configs", action="store_true",
+                    help="time only the chosen workload (by default a 1-GPU run also times C1, C2, C3, C5 "
+                         "routed and C5 forced-8 and reports them under configs)")
     ap.add_argument("--decode-batch", type=int, default=0, help="override the workload's batch (C5 sweep)")
     ap.add_argument("--ablation", default="none", choices=["none", "no_gather", "dense_cache"],
                     help="no_gather: all rows every loop, exited rows masked (no gather of Eq. 6); "
