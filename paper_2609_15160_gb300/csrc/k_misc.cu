@@ -216,12 +216,34 @@ __global__ void __launch_bounds__(256) k_final(ModelDims md, StepDev s, const fl
   pdl_wait();
   pdl_trigger();
   const int b = blockIdx.x;
-  const float* h = s.H + (size_t)b * md.d;
+  // the row (d <= 8192, a multiple of 64) is read once into registers, 16 bytes per load
+  const float4* h4 = reinterpret_cast<const float4*>(s.H + (size_t)b * md.d);
+  const float4* g4 = reinterpret_cast<const float4*>(gain);
+  const int d4 = md.d / 4;
+  float4 v[8];
   float ss = 0.f;
-  for (int i = threadIdx.x; i < md.d; i += blockDim.x) ss += h[i] * h[i];
+#pragma unroll
+  for (int c = 0; c < 8; ++c) {
+    const int i = threadIdx.x + c * blockDim.x;
+    if (i < d4) {
+      v[c] = h4[i];
+      ss += v[c].x * v[c].x + v[c].y * v[c].y + v[c].z * v[c].z + v[c].w * v[c].w;
+    }
+  }
   ss = block_sum(ss);
   const float inv = rsqrtf(ss / (float)md.d + md.eps);
-  for (int i = threadIdx.x; i < md.d; i += blockDim.x) Xf[(size_t)b * md.d + i] = from_f32<T>(h[i] * inv * gain[i]);
+  T* xr = Xf + (size_t)b * md.d;
+#pragma unroll
+  for (int c = 0; c < 8; ++c) {
+    const int i = threadIdx.x + c * blockDim.x;
+    if (i < d4) {
+      const float4 g = g4[i];
+      xr[4 * i + 0] = from_f32<T>(v[c].x * inv * g.x);
+      xr[4 * i + 1] = from_f32<T>(v[c].y * inv * g.y);
+      xr[4 * i + 2] = from_f32<T>(v[c].z * inv * g.z);
+      xr[4 * i + 3] = from_f32<T>(v[c].w * inv * g.w);
+    }
+  }
   if (threadIdx.x < md.M) {
     // every loop cache the token wrote to grows by one (all of them without recursion-wise caches,
     // where the loops it skipped hold a masked slot)

@@ -1,12 +1,13 @@
 // Token-choice router and active-set compaction (T-LoopFormer Sec. 3.2, Eq. 2-6).
 //
-// k_router: one warp per token. h^(0) = E[x] is written to the float32
-// residual stream H, RMSNorm (no gain) is applied, the M router logits
-// z = W_r x + b_r are reduced across the warp, and the loop count m and its
-// decision margin are taken in float32 (ARGMAX or SURVIVAL rule, see tlf.h).
+// k_router: four warps per token, each over a quarter of the row. h^(0) = E[x]
+// is written to the float32 residual stream H, RMSNorm (no gain) is applied,
+// the M router logits z = W_r x + b_r are reduced across the warps, and the
+// loop count m and its decision margin are taken in float32 (ARGMAX or
+// SURVIVAL rule, see tlf.h).
 // The same kernel applies the page-table updates the host queued for the step.
 //
-// k_plan: one CTA. For every loop r it builds A_r = {b : m_b >= r} in
+// k_plan: one CTA per loop r. It builds A_r = {b : m_b >= r} in
 // increasing b with a warp ballot plus a block prefix scan, the page, slot
 // and position of each active token's new loop-r cache entry (read by the
 // QKV epilogue that appends k, v), and the work plan of the decode attention
@@ -64,6 +65,10 @@ __device__ __forceinline__ void router_decide(const ModelDims& md, const float z
   }
 }
 
+// Warps per token of k_router: each reads a quarter of the row, so the dependent chain of
+// 16-byte loads per lane is a quarter as long; a CTA of 8 warps serves two tokens.
+constexpr int RT_WPT = 4;
+
 template <typename T>
 __global__ void __launch_bounds__(256) k_router(ModelDims md, StepDev s, int B, const T* __restrict__ emb,
                                                 const T* __restrict__ rw, const float* __restrict__ rb,
@@ -75,48 +80,74 @@ __global__ void __launch_bounds__(256) k_router(ModelDims md, StepDev s, int B, 
     const PageUpdate p = upd[u];
     s.page_table[p.index] = p.page;
   }
+  __shared__ float part_sum[8][17];  // per warp: sum of squares, then the M dot products
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int b = blockIdx.x * 8 + warp;
-  if (b >= B) return;
+  const int quarter = warp % RT_WPT;
+  const int b = blockIdx.x * (8 / RT_WPT) + warp / RT_WPT;
   const int d = md.d, M = md.M;
-  int tok = s.tokens[b];
-  if (tok < 0 || tok >= md.V) {
-    if (lane == 0) atomicOr(s.err, DEVERR_INDEX);
-    tok = 0;
-  }
-  // One pass over 16-byte chunks: each chunk of E[x] is loaded once, written to
-  // the residual stream, squared into the norm, and dotted with all M router rows;
-  // the RMSNorm scale (a per-row scalar) multiplies the dot products afterwards.
-  constexpr int VEC = Vec16<T>::N;
-  const T* e = emb + (size_t)tok * d;
-  float* h = s.H + (size_t)b * d;
-  float ss = 0.f, dot[16];
+  if (b < B) {
+    int tok = s.tokens[b];
+    if (tok < 0 || tok >= md.V) {
+      if (lane == 0 && quarter == 0) atomicOr(s.err, DEVERR_INDEX);
+      tok = 0;
+    }
+    // One pass over 16-byte chunks: each chunk of E[x] is loaded once, written to the residual
+    // stream, squared into the norm, and dotted with all M router rows; the RMSNorm scale (a
+    // per-row scalar) multiplies the dot products afterwards.
+    constexpr int VEC = Vec16<T>::N;
+    const T* e = emb + (size_t)tok * d;
+    float* h = s.H + (size_t)b * d;
+    float ss = 0.f, dot[16];
 #pragma unroll
-  for (int l = 0; l < 16; ++l) dot[l] = 0.f;
-  for (int c = lane; c < d / VEC; c += 32) {
-    float x[VEC];
-    Vec16<T>::load(e + c * VEC, x);
+    for (int l = 0; l < 16; ++l) dot[l] = 0.f;
+#pragma unroll 2
+    for (int c = quarter * 32 + lane; c < d / VEC; c += 32 * RT_WPT) {
+      float x[VEC];
+      Vec16<T>::load(e + c * VEC, x);
 #pragma unroll
-    for (int u = 0; u < VEC; u += 4)
-      *reinterpret_cast<float4*>(h + c * VEC + u) = make_float4(x[u], x[u + 1], x[u + 2], x[u + 3]);
+      for (int u = 0; u < VEC; u += 4)
+        *reinterpret_cast<float4*>(h + c * VEC + u) = make_float4(x[u], x[u + 1], x[u + 2], x[u + 3]);
 #pragma unroll
-    for (int u = 0; u < VEC; ++u) ss = fmaf(x[u], x[u], ss);
+      for (int u = 0; u < VEC; ++u) ss = fmaf(x[u], x[u], ss);
 #pragma unroll
-    for (int l = 0; l < 16; ++l) {
-      if (l < M) {
-        float w[VEC];
-        Vec16<T>::load(rw + (size_t)l * d + c * VEC, w);
+      for (int l = 0; l < 16; ++l) {
+        if (l < M) {
+          float w[VEC];
+          Vec16<T>::load(rw + (size_t)l * d + c * VEC, w);
 #pragma unroll
-        for (int u = 0; u < VEC; ++u) dot[l] = fmaf(x[u], w[u], dot[l]);
+          for (int u = 0; u < VEC; ++u) dot[l] = fmaf(x[u], w[u], dot[l]);
+        }
       }
     }
+    ss = warp_sum(ss);
+#pragma unroll
+    for (int l = 0; l < 16; ++l)
+      if (l < M) dot[l] = warp_sum(dot[l]);
+    if (lane == 0) {
+      part_sum[warp][0] = ss;
+#pragma unroll
+      for (int l = 0; l < 16; ++l)
+        if (l < M) part_sum[warp][1 + l] = dot[l];
+    }
   }
-  ss = warp_sum(ss);
+  __syncthreads();
+  if (b >= B || quarter != 0) return;
+  // the token's first warp adds the quarters (in a fixed order) and takes the decision
+  const int w0 = warp;
+  float ss = 0.f;
+#pragma unroll
+  for (int q = 0; q < RT_WPT; ++q) ss += part_sum[w0 + q][0];
   const float inv = rsqrtf(ss / (float)d + md.eps);
-
   float z[16];
 #pragma unroll
-  for (int l = 0; l < 16; ++l) z[l] = (l < M) ? warp_sum(dot[l]) * inv + rb[l] : -INFINITY;
+  for (int l = 0; l < 16; ++l) {
+    float t = 0.f;
+    if (l < M) {
+#pragma unroll
+      for (int q = 0; q < RT_WPT; ++q) t += part_sum[w0 + q][1 + l];
+    }
+    z[l] = (l < M) ? t * inv + rb[l] : -INFINITY;
+  }
 
   int m;
   float margin;
@@ -250,6 +281,7 @@ __device__ int block_exclusive_scan(int v, int* total) {
   return excl;
 }
 
+// One CTA per loop r (the loops' lists and plans are independent), one thread per batch row.
 __global__ void __launch_bounds__(256) k_plan(ModelDims md, StepDev s, int B) {
   pdl_wait();
   pdl_trigger();
@@ -259,11 +291,13 @@ __global__ void __launch_bounds__(256) k_plan(ModelDims md, StepDev s, int B) {
   const int slot = (b < B) ? s.slots[b] : 0;
   const int maxB = md.max_batch, M = md.M, ps = md.page_size;
   // attention merge tickets start at zero every step
-  for (int i = b; i < maxB * md.Hkv; i += blockDim.x) s.cnt[i] = 0;
+  if (blockIdx.x == 0)
+    for (int i = b; i < maxB * md.Hkv; i += blockDim.x) s.cnt[i] = 0;
   // without the gather (an ablation), every row of the step is listed at every loop that runs
   const bool all_rows = md.ablation == TLF_ABLATION_NO_GATHER;
   const bool dense = md.ablation == TLF_ABLATION_DENSE_CACHE;
-  for (int r = 0; r < M; ++r) {
+  {
+    const int r = blockIdx.x;
     const bool active = mb > r;
     // compaction: ballot gives each active lane its rank in the warp, the block scan the warp offsets
     const unsigned ball = __ballot_sync(0xffffffffu, active);
@@ -345,7 +379,7 @@ void launch_router(const ModelDims& md, const StepDev& s, int B, const void* emb
                router_b1, (const float*)router_w, router_b, upd, n_upd);
     return;
   }
-  const int grid = (B + 7) / 8;
+  const int grid = (B + 8 / RT_WPT - 1) / (8 / RT_WPT);
   if (md.dtype == 1)
     launch_k(k_router<bf16>, grid, 256, 0, st, md, s, B, (const bf16*)emb, (const bf16*)router_w, router_b, upd,
              n_upd);
@@ -355,7 +389,7 @@ void launch_router(const ModelDims& md, const StepDev& s, int B, const void* emb
 }
 
 void launch_plan(const ModelDims& md, const StepDev& s, int B, cudaStream_t st) {
-  launch_k(k_plan, 1, 256, 0, st, md, s, B);
+  launch_k(k_plan, md.M, 256, 0, st, md, s, B);
 }
 
 }  // namespace tlf
