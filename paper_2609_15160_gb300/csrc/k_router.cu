@@ -24,17 +24,22 @@ __device__ __forceinline__ void router_decide(const ModelDims& md, const float z
   const int M = md.M;
   m = 1;
   if (md.exit_rule == 0) {
-    // ARGMAX: first maximum wins (ties go to the smaller depth)
+    // ARGMAX: first maximum wins (ties go to the smaller depth); indices stay compile-time
+    // constants so z lives in registers
     int top = 0;
+    float best = z[0];
 #pragma unroll
     for (int l = 1; l < 16; ++l)
-      if (l < M && z[l] > z[top]) top = l;
+      if (l < M && z[l] > best) {
+        best = z[l];
+        top = l;
+      }
     float second = -INFINITY;
 #pragma unroll
     for (int l = 0; l < 16; ++l)
       if (l < M && l != top) second = fmaxf(second, z[l]);
     m = top + 1;
-    margin = z[top] - second;  // +inf when M == 1
+    margin = best - second;  // +inf when M == 1
   } else {
     // SURVIVAL (Eq. 2-5): softmax, suffix sums p^(i), m = max{i : p^(i) > threshold}
     float mx = z[0];
@@ -59,8 +64,12 @@ __device__ __forceinline__ void router_decide(const ModelDims& md, const float z
 #pragma unroll
     for (int l = 0; l < 16; ++l)
       if (l < M && p[l] > md.threshold) m = l + 1;
-    const float pm = p[m - 1];
-    const float pnext = (m < M) ? p[m] : 0.f;
+    float pm = 0.f, pnext = 0.f;  // p^(m) and p^(m+1) (0 past M)
+#pragma unroll
+    for (int l = 0; l < 16; ++l) {
+      if (l == m - 1) pm = p[l];
+      if (l == m && l < M) pnext = p[l];
+    }
     margin = fminf(pm - md.threshold, md.threshold - pnext);
   }
 }
