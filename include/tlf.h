@@ -183,7 +183,7 @@ int64_t tlf_page_bytes(const tlf_config* cfg);
  *
  * Environment switches select equivalent comparison paths, each covered by
  * the GPU tests. The first two change only how kernels are launched, and the
- * results are bit-identical; the last two change rounding, within the logits
+ * results are bit-identical; the others change rounding, within the logits
  * tolerance.
  *   TLF_NO_GRAPH=1       launch each step's kernels directly instead of
  *                        replaying a captured CUDA graph (read here)
@@ -193,7 +193,12 @@ int64_t tlf_page_bytes(const tlf_config* cfg);
  *                        of split across the neighbouring GEMMs (read here)
  *   TLF_NO_OPERAND_LO=1  one bf16 plane for the decode GEMMs' activation
  *                        operands instead of hi + lo (two-term) planes (read
- *                        here) */
+ *                        here)
+ *   TLF_PF_ATTN_V1=1     prefill attention with every thread staging and
+ *                        re-laying out each K/V page instead of the
+ *                        warp-specialised kernel that loads pages with a
+ *                        tensor map (read here; same arithmetic, different
+ *                        rounding order of the row sums) */
 int tlf_create(const tlf_config* cfg, const tlf_weights* w, tlf_ctx** out);
 
 /* Free every device and host resource of the context: the weights, the

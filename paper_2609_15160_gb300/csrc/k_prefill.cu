@@ -578,6 +578,329 @@ __global__ void __launch_bounds__(PFT_THREADS) k_pf_attn_tc(ModelDims md, Prefil
   if (warp == 0) tmem_dealloc(tmem, Sh::TMEM_COLS);
 }
 
+// ----------------------------------------------------------------------------
+// Warp-specialised tensor-core causal attention of a chunk (bf16, head_dim 64 or 128)
+// ----------------------------------------------------------------------------
+// Same work split as k_pf_attn_tc (one CTA per sequence, block of QT = 128/G queries and kv head;
+// the 128 MMA rows are query * G + head; cache pages of 64 slots), with the roles split across
+// warps so that no block-wide barrier sits in the page loop:
+//   warp 4      TMA producer: the K and V segments of every page, straight from the paged pool
+//               through a 3-D tensor map (128-byte swizzle), into two-deep K and V rings;
+//   warp 5      MMA issuer: S(p) = Q K(p)^T into one of two TMEM buffers (q as bf16 hi + lo terms,
+//               so the scores keep q's float32 precision), then O += P(p-1) V(p-1) with V taken as
+//               an MN-major operand (no transpose);
+//   warps 0-3   softmax, one thread per row: read the row of S(p) from TMEM, mask causally by cache
+//               slot, keep the running maximum (refreshed lazily: O is rescaled in TMEM only when a
+//               row's maximum grows by more than 8 in base 2) and sum in float32, and write P(p) in
+//               bf16 to one of two shared-memory buffers; at the end they normalise O and store it.
+// mbarriers connect the roles (ring full / empty, S full / free, P full / free); every wait is
+// bounded. Slots past the block's last query in its last page hold finite values (the pool is
+// zeroed when created and only ever holds finite entries), which the mask turns into P = 0.
+constexpr int PFW_THREADS = 192;
+
+template <int HD>
+struct PfWsShape {
+  static constexpr int ATOMS = HD / 64;                // 128-byte atom columns of a row
+  static constexpr int Q_BYTES = 128 * HD * 2;         // one of the hi / lo Q tiles [128][HD]
+  static constexpr int QCOL = 128 * 128;               // bytes of one atom column of a Q tile
+  static constexpr int KV_BYTES = 64 * HD * 2;         // a K (or V) stage: [64 keys][HD]
+  static constexpr int KVCOL = 64 * 128;               // bytes of one atom column of a stage
+  static constexpr int NST = 2;                        // ring depth
+  static constexpr int P_BYTES = 128 * 64 * 2;         // a P buffer [128][64 keys]
+  static constexpr int OFF_QHI = 0;
+  static constexpr int OFF_QLO = OFF_QHI + Q_BYTES;
+  static constexpr int OFF_K = OFF_QLO + Q_BYTES;
+  static constexpr int OFF_V = OFF_K + NST * KV_BYTES;
+  static constexpr int OFF_P = OFF_V + NST * KV_BYTES;
+  static constexpr int OFF_BAR = OFF_P + 2 * P_BYTES;
+  static constexpr int NBAR = 4 * NST + 8;
+  static constexpr int BYTES = OFF_BAR + NBAR * 8 + 16 + 1024;  // barriers, TMEM slot, alignment slack
+  static constexpr uint32_t TMEM_COLS = 256;          // S buffers in columns 0..127, O in 128..128+HD
+};
+
+template <int HD, int G>
+__global__ void __launch_bounds__(PFW_THREADS) k_pf_attn_ws(ModelDims md, PrefillDev p, StepDev s, int r, int j,
+                                                             const float* __restrict__ Q, bf16* __restrict__ O,
+                                                             const __grid_constant__ CUtensorMap pool_map) {
+  using Sh = PfWsShape<HD>;
+  constexpr int QT = 128 / G, NST = Sh::NST;
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* sm = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+  uint64_t* bars = reinterpret_cast<uint64_t*>(sm + Sh::OFF_BAR);
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + Sh::NBAR);
+  auto bar = [&](int i) { return smem_u32(&bars[i]); };
+  // K full / empty, V full / empty (NST each), then S full x2, S free x2, P full x2, P free x2
+  auto k_full = [&](int st) { return bar(st); };
+  auto k_empty = [&](int st) { return bar(NST + st); };
+  auto v_full = [&](int st) { return bar(2 * NST + st); };
+  auto v_empty = [&](int st) { return bar(3 * NST + st); };
+  auto s_full = [&](int b) { return bar(4 * NST + b); };
+  auto s_free = [&](int b) { return bar(4 * NST + 2 + b); };
+  auto p_full = [&](int b) { return bar(4 * NST + 4 + b); };
+  auto p_free = [&](int b) { return bar(4 * NST + 6 + b); };
+
+  pdl_wait();
+  pdl_trigger();
+  const int S = p.S;
+  const int* tbase = p.tile_base + r * (p.Smax + 1);
+  const int tile = blockIdx.x, kvh = blockIdx.y;
+  if (tile >= tbase[S]) return;
+  int lo = 0, hi = S;  // sequence: largest sq with tbase[sq] <= tile
+  while (hi - lo > 1) {
+    const int mid = (lo + hi) >> 1;
+    if (tbase[mid] <= tile) lo = mid; else hi = mid;
+  }
+  const int sq = lo, qb = tile - tbase[sq];
+  const int cnt = p.cnt[r * p.Smax + sq], first = p.first[r * p.Smax + sq], s0 = p.s0[r * p.Smax + sq];
+  const int slot = p.seq_slot[sq];
+  const int q0 = qb * QT, nq = min(QT, cnt - q0);
+  const int last = s0 + q0 + nq - 1;  // cache slot of the block's last query
+  const int npages = last / 64 + 1;
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  const int* ptab = s.page_table + ((size_t)slot * md.M + r) * md.max_pages;
+
+  if (tid == 0) {
+    for (int i = 0; i < NST; ++i) {
+      mbar_init(k_full(i), 1);
+      mbar_init(k_empty(i), 1);
+      mbar_init(v_full(i), 1);
+      mbar_init(v_empty(i), 1);
+    }
+    for (int b = 0; b < 2; ++b) {
+      mbar_init(s_full(b), 1);
+      mbar_init(s_free(b), 4);
+      mbar_init(p_full(b), 4);
+      mbar_init(p_free(b), 1);
+    }
+    fence_barrier_init();
+    prefetch_tensormap(&pool_map);
+  }
+  if (warp == 5) {
+    tmem_alloc(smem_u32(tmem_slot), Sh::TMEM_COLS);
+    tmem_relinquish();
+  }
+  // Q tile: row = query * G + head, as hi and lo bf16 parts (zeros past the block's queries)
+  for (int e = tid; e < 128 * (HD / 8); e += PFW_THREADS) {
+    const int qr = e / (HD / 8), c = e % (HD / 8);
+    const int qq = qr / G, gg = qr % G;
+    float x[8];
+    if (qq < nq) {
+      const float4* q4 = reinterpret_cast<const float4*>(Q + ((size_t)(first + q0 + qq) * md.Hq + kvh * G + gg) * HD);
+      const float4 a = q4[2 * c], b = q4[2 * c + 1];
+      x[0] = a.x; x[1] = a.y; x[2] = a.z; x[3] = a.w; x[4] = b.x; x[5] = b.y; x[6] = b.z; x[7] = b.w;
+    } else {
+#pragma unroll
+      for (int u = 0; u < 8; ++u) x[u] = 0.f;
+    }
+    uint32_t h[4], l[4];
+#pragma unroll
+    for (int u = 0; u < 4; ++u) {
+      const float a0 = __bfloat162float(__float2bfloat16_rn(x[2 * u]));
+      const float a1 = __bfloat162float(__float2bfloat16_rn(x[2 * u + 1]));
+      h[u] = pack_bf16(a0, a1);
+      l[u] = pack_bf16(x[2 * u] - a0, x[2 * u + 1] - a1);
+    }
+    const uint32_t off = (c / 8) * Sh::QCOL + sw128_off(qr, c % 8);
+    *reinterpret_cast<uint4*>(sm + Sh::OFF_QHI + off) = make_uint4(h[0], h[1], h[2], h[3]);
+    *reinterpret_cast<uint4*>(sm + Sh::OFF_QLO + off) = make_uint4(l[0], l[1], l[2], l[3]);
+  }
+  fence_proxy_async_smem();
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = *tmem_slot;
+  constexpr uint32_t OCOL = 128;  // first TMEM column of O
+  volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
+  if (tid == 0) *abort_flag = 0;
+  __syncthreads();
+  // a bounded wait; once any role has given up, the others skip their waits and wind down
+  auto wait = [&](uint32_t b, uint32_t parity) {
+    if (*abort_flag) return false;
+    if (!mbar_wait(b, parity, s.err)) {
+      *abort_flag = 1;
+      return false;
+    }
+    return true;
+  };
+
+  if (warp == 4) {
+    // ---------------- TMA producer ----------------
+    if (lane == 0) {
+      const int rowK = ((j * 2 + 0) * md.Hkv + kvh) * 64, rowV = ((j * 2 + 1) * md.Hkv + kvh) * 64;
+      for (int pg = 0; pg < npages; ++pg) {
+        const int st = pg % NST;
+        const uint32_t par = (uint32_t)((pg / NST) - 1) & 1u;
+        int page = ptab[pg];
+        const bool okp = page >= 0 && page < md.n_pages;
+        if (!okp) atomicOr(s.err, DEVERR_INDEX);
+        if (pg >= NST && !wait(k_empty(st), par)) break;
+        if (okp) {
+          mbar_arrive_expect_tx(k_full(st), Sh::KV_BYTES);
+#pragma unroll
+          for (int a = 0; a < Sh::ATOMS; ++a)
+            tma_load_3d(smem_u32(sm + Sh::OFF_K + st * Sh::KV_BYTES + a * Sh::KVCOL), &pool_map, a * 64, rowK, page,
+                        k_full(st));
+        } else {
+          mbar_arrive(k_full(st));  // complete the phase without data
+        }
+        if (pg >= NST && !wait(v_empty(st), par)) break;
+        if (okp) {
+          mbar_arrive_expect_tx(v_full(st), Sh::KV_BYTES);
+#pragma unroll
+          for (int a = 0; a < Sh::ATOMS; ++a)
+            tma_load_3d(smem_u32(sm + Sh::OFF_V + st * Sh::KV_BYTES + a * Sh::KVCOL), &pool_map, a * 64, rowV, page,
+                        v_full(st));
+        } else {
+          mbar_arrive(v_full(st));
+        }
+      }
+    }
+  } else if (warp == 5) {
+    // ---------------- MMA issuer ----------------
+    if (lane == 0) {
+      constexpr uint32_t IDS = idesc_bf16_f32(128, 64), IDO = idesc_bf16_f32_bmn(128, HD);
+      auto issue_pv = [&](int q) {  // O += P(q) V(q)
+        const int bq = q & 1, st = q % NST;
+        if (!wait(p_full(bq), (uint32_t)(q >> 1) & 1u) || !wait(v_full(st), (uint32_t)(q / NST) & 1u)) return false;
+        tc_fence_after();
+        const uint32_t pa = smem_u32(sm + Sh::OFF_P + bq * Sh::P_BYTES);
+        const uint32_t vb = smem_u32(sm + Sh::OFF_V + st * Sh::KV_BYTES);
+#pragma unroll
+        for (int k = 0; k < 4; ++k)  // K = 16 keys per MMA: +32 B in P's rows, +2048 B (16 rows) in V
+          tc_mma_f16(tmem + OCOL, smem_desc_sw128(pa) + 2 * k, smem_desc_sw128_mn(vb + 2048u * k, Sh::KVCOL), IDO,
+                     (q > 0 || k > 0) ? 1u : 0u);
+        tc_commit(p_free(bq));
+        tc_commit(v_empty(st));
+        return true;
+      };
+      bool ok = true;
+      for (int pg = 0; pg < npages && ok; ++pg) {
+        const int b = pg & 1, st = pg % NST;
+        if (!wait(k_full(st), (uint32_t)(pg / NST) & 1u)) break;
+        if (pg >= 2 && !wait(s_free(b), (uint32_t)((pg - 2) >> 1) & 1u)) break;
+        tc_fence_after();
+        const uint32_t kb = smem_u32(sm + Sh::OFF_K + st * Sh::KV_BYTES);
+#pragma unroll
+        for (int kc = 0; kc < Sh::ATOMS; ++kc)
+#pragma unroll
+          for (int k = 0; k < 4; ++k) {  // K = 16 per MMA: +32 bytes (encoded +2) inside the atom column
+            const uint64_t db = smem_desc_sw128(kb + kc * Sh::KVCOL) + 2 * k;
+            const uint32_t d = tmem + 64u * (uint32_t)b;
+            tc_mma_f16(d, smem_desc_sw128(smem_u32(sm + Sh::OFF_QHI + kc * Sh::QCOL)) + 2 * k, db, IDS,
+                       (kc | k) ? 1u : 0u);
+            tc_mma_f16(d, smem_desc_sw128(smem_u32(sm + Sh::OFF_QLO + kc * Sh::QCOL)) + 2 * k, db, IDS, 1u);
+          }
+        tc_commit(s_full(b));
+        tc_commit(k_empty(st));
+        if (pg >= 1) ok = issue_pv(pg - 1);
+      }
+      if (ok) issue_pv(npages - 1);
+    }
+  } else {
+    // ---------------- softmax: thread = MMA row = TMEM lane ----------------
+    const int row = warp * 32 + lane;
+    const uint32_t t_row = tmem + ((uint32_t)(warp * 32) << 16);
+    const int qi = row / G, g = row % G;
+    const bool row_ok = qi < nq;
+    const int qslot = s0 + q0 + qi;  // cache slot of this row's query
+    const float scale = 1.4426950408889634f * rsqrtf((float)HD);
+    float m_run = -INFINITY, l_run = 0.f;
+    bool ok = true;
+    // waits taken by the whole warp: the TMEM accesses after them are warp-collective
+    auto wait_w = [&](uint32_t bq, uint32_t parity) { return __all_sync(0xffffffffu, wait(bq, parity)); };
+    for (int pg = 0; pg < npages && ok; ++pg) {
+      const int b = pg & 1;
+      if (!wait_w(s_full(b), (uint32_t)(pg >> 1) & 1u)) { ok = false; break; }
+      tc_fence_after();
+      float sc[64];
+      tmem_ld_32(t_row + 64u * (uint32_t)b, sc);
+      tmem_ld_32(t_row + 64u * (uint32_t)b + 32u, sc + 32);
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(s_free(b));
+      const int kb = pg * 64;  // cache slot of column 0
+      float pm = -INFINITY;
+      if (row_ok && kb + 63 <= qslot) {  // every key visible
+#pragma unroll
+        for (int c = 0; c < 64; ++c) {
+          sc[c] *= scale;
+          pm = fmaxf(pm, sc[c]);
+        }
+      } else if (!row_ok || kb > qslot) {  // none visible
+#pragma unroll
+        for (int c = 0; c < 64; ++c) sc[c] = -INFINITY;
+      } else {  // the diagonal: causal by cache slot
+#pragma unroll
+        for (int c = 0; c < 64; ++c) {
+          sc[c] = kb + c <= qslot ? sc[c] * scale : -INFINITY;
+          pm = fmaxf(pm, sc[c]);
+        }
+      }
+      // lazy maximum: O is rescaled only when a row's maximum grows by more than 8, after the
+      // P V product before has landed (warp-uniform TMEM access)
+      const bool grow = pm > m_run + 8.f;
+      const float cr = grow ? exp2f(m_run - pm) : 1.f;  // 0 when m_run was -inf
+      if (pg > 0 && __any_sync(0xffffffffu, grow)) {
+        if (!wait_w(p_free((pg - 1) & 1), (uint32_t)((pg - 1) >> 1) & 1u)) { ok = false; break; }
+        tc_fence_after();
+#pragma unroll
+        for (int c0 = 0; c0 < HD; c0 += 16) {
+          float o[16];
+          tmem_ld_16(t_row + OCOL + (uint32_t)c0, o);
+#pragma unroll
+          for (int i = 0; i < 16; ++i) o[i] *= cr;
+          tmem_st_16(t_row + OCOL + (uint32_t)c0, o);
+        }
+        tc_fence_before();
+      }
+      if (grow) {
+        l_run *= cr;
+        m_run = pm;
+      }
+      uint32_t pk[32];
+      float psum = 0.f;
+#pragma unroll
+      for (int c = 0; c < 64; c += 2) {
+        const float p0 = sc[c] == -INFINITY ? 0.f : ex2_approx(sc[c] - m_run);
+        const float p1 = sc[c + 1] == -INFINITY ? 0.f : ex2_approx(sc[c + 1] - m_run);
+        psum += p0 + p1;
+        pk[c / 2] = pack_bf16(p0, p1);
+      }
+      l_run += psum;
+      // P buffer b was last read by P V of page pg - 2
+      if (pg >= 2 && !wait_w(p_free(b), (uint32_t)((pg - 2) >> 1) & 1u)) { ok = false; break; }
+      uint8_t* pb = sm + Sh::OFF_P + b * Sh::P_BYTES;
+#pragma unroll
+      for (int q = 0; q < 8; ++q)
+        *reinterpret_cast<uint4*>(pb + sw128_off(row, q)) = make_uint4(pk[4 * q], pk[4 * q + 1], pk[4 * q + 2], pk[4 * q + 3]);
+      fence_proxy_async_smem();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(p_full(b));
+    }
+    // the last P V product, then O / l out
+    if (ok && wait_w(p_free((npages - 1) & 1), (uint32_t)((npages - 1) >> 1) & 1u)) {
+      tc_fence_after();
+      const float inv_l = l_run > 0.f ? 1.f / l_run : 0.f;
+      bf16* orow = O + (size_t)(first + q0 + qi) * md.q_dim + (kvh * G + g) * HD;
+#pragma unroll
+      for (int c0 = 0; c0 < HD; c0 += 16) {
+        float o[16];
+        tmem_ld_16(t_row + OCOL + (uint32_t)c0, o);
+        if (row_ok) {
+          uint32_t w[8];
+#pragma unroll
+          for (int i = 0; i < 8; ++i) w[i] = pack_bf16(o[2 * i] * inv_l, o[2 * i + 1] * inv_l);
+          *reinterpret_cast<uint4*>(orow + c0) = make_uint4(w[0], w[1], w[2], w[3]);
+          *reinterpret_cast<uint4*>(orow + c0 + 8) = make_uint4(w[4], w[5], w[6], w[7]);
+        }
+      }
+    }
+  }
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 5) tmem_dealloc(tmem, Sh::TMEM_COLS);
+}
+
 __global__ void k_pf_len(ModelDims md, PrefillDev p) {
   pdl_wait();
   pdl_trigger();
@@ -615,6 +938,19 @@ static void pf_attn_tc_launch(const ModelDims& md, const PrefillDev& p, const St
   launch_k(k_pf_attn_tc<HD, G>, dim3(tiles_bound, md.Hkv), PFT_THREADS, smem, st, md, p, s, r, j, Q, (bf16*)O);
 }
 
+template <int HD, int G>
+static void pf_attn_ws_launch(const ModelDims& md, const PrefillDev& p, const StepDev& s, int r, int j,
+                              const float* Q, void* O, int tiles_bound, cudaStream_t st, const CUtensorMap* pool_map) {
+  static bool attr = false;
+  constexpr int smem = PfWsShape<HD>::BYTES;
+  if (!attr) {
+    cudaFuncSetAttribute(k_pf_attn_ws<HD, G>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+    attr = true;
+  }
+  launch_k(k_pf_attn_ws<HD, G>, dim3(tiles_bound, md.Hkv), PFW_THREADS, smem, st, md, p, s, r, j, Q, (bf16*)O,
+           *pool_map);
+}
+
 // Tensor-core kernel for head_dim 64 and 128 (128-byte rows for the swizzled operand tiles); the
 // CUDA-core kernel for head_dim 32.
 static bool pf_attn_uses_tc(const ModelDims& md) { return md.hd == 64 || md.hd == 128; }
@@ -622,8 +958,17 @@ static bool pf_attn_uses_tc(const ModelDims& md) { return md.hd == 64 || md.hd =
 int pf_attn_qblock(const ModelDims& md) { return pf_attn_uses_tc(md) ? 128 / (md.Hq / md.Hkv) : PF_QB; }
 
 void launch_pf_attn(const ModelDims& md, const PrefillDev& p, const StepDev& s, int r, int j, const float* Q,
-                    void* O, int tiles_bound, cudaStream_t st) {
+                    void* O, int tiles_bound, cudaStream_t st, const CUtensorMap* pool_map) {
   const int G = md.Hq / md.Hkv;
+  if (pool_map && (md.hd == 64 || md.hd == 128)) {
+    if (md.hd == 128 && G == 1) pf_attn_ws_launch<128, 1>(md, p, s, r, j, Q, O, tiles_bound, st, pool_map);
+    else if (md.hd == 128 && G == 2) pf_attn_ws_launch<128, 2>(md, p, s, r, j, Q, O, tiles_bound, st, pool_map);
+    else if (md.hd == 128 && G == 4) pf_attn_ws_launch<128, 4>(md, p, s, r, j, Q, O, tiles_bound, st, pool_map);
+    else if (md.hd == 64 && G == 1) pf_attn_ws_launch<64, 1>(md, p, s, r, j, Q, O, tiles_bound, st, pool_map);
+    else if (md.hd == 64 && G == 2) pf_attn_ws_launch<64, 2>(md, p, s, r, j, Q, O, tiles_bound, st, pool_map);
+    else pf_attn_ws_launch<64, 4>(md, p, s, r, j, Q, O, tiles_bound, st, pool_map);
+    return;
+  }
   if (md.hd == 128 && G == 1) pf_attn_tc_launch<128, 1>(md, p, s, r, j, Q, O, tiles_bound, st);
   else if (md.hd == 128 && G == 2) pf_attn_tc_launch<128, 2>(md, p, s, r, j, Q, O, tiles_bound, st);
   else if (md.hd == 128 && G == 4) pf_attn_tc_launch<128, 4>(md, p, s, r, j, Q, O, tiles_bound, st);

