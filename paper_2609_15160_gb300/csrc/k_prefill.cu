@@ -643,8 +643,11 @@ __global__ void __launch_bounds__(PFW_THREADS) k_pf_attn_ws(ModelDims md, Prefil
   pdl_trigger();
   const int S = p.S;
   const int* tbase = p.tile_base + r * (p.Smax + 1);
-  const int tile = blockIdx.x, kvh = blockIdx.y;
-  if (tile >= tbase[S]) return;
+  // 1-D grid, kv head fastest and query blocks in reverse order: the blocks with the most pages
+  // (the last queries of a sequence) are dispatched first, so the last wave holds short ones
+  const int ntiles = tbase[S];
+  const int kvh = blockIdx.x % md.Hkv, tile = ntiles - 1 - (int)(blockIdx.x / md.Hkv);
+  if (tile < 0) return;
   int lo = 0, hi = S;  // sequence: largest sq with tbase[sq] <= tile
   while (hi - lo > 1) {
     const int mid = (lo + hi) >> 1;
@@ -947,7 +950,7 @@ static void pf_attn_ws_launch(const ModelDims& md, const PrefillDev& p, const St
     cudaFuncSetAttribute(k_pf_attn_ws<HD, G>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
     attr = true;
   }
-  launch_k(k_pf_attn_ws<HD, G>, dim3(tiles_bound, md.Hkv), PFW_THREADS, smem, st, md, p, s, r, j, Q, (bf16*)O,
+  launch_k(k_pf_attn_ws<HD, G>, dim3(tiles_bound * md.Hkv), PFW_THREADS, smem, st, md, p, s, r, j, Q, (bf16*)O,
            *pool_map);
 }
 

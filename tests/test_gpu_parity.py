@@ -351,6 +351,15 @@ def test_head_dims(tlf, hd):
     _prefill_decode_compare(tlf, _small(head_dim=hd, n_heads=4, n_kv_heads=2, d_model=256), [66, 3], steps=2)
 
 
+@pytest.mark.parametrize("hd,gqa", [(64, (4, 4)), (128, (8, 2))])
+def test_thread_staged_prefill_attention_path(tlf, monkeypatch, hd, gqa):
+    """The prefill attention that stages and re-lays out every K/V page with its threads
+    (TLF_PF_ATTN_V1=1), the comparison path of the tensor-map kernel, on multi-page prompts."""
+    monkeypatch.setenv("TLF_PF_ATTN_V1", "1")
+    m = _small(head_dim=hd, n_heads=gqa[0], n_kv_heads=gqa[1], d_model=256)
+    _prefill_decode_compare(tlf, m, [300, 65, 1], steps=2)
+
+
 def test_every_token_exits_after_one_loop(tlf):
     """Deeper loops have no active token (device-side counts are zero)."""
     _prefill_decode_compare(tlf, _small(), [30, 65], steps=3, forced_mode=1)
