@@ -584,8 +584,9 @@ __global__ void __launch_bounds__(PFT_THREADS) k_pf_attn_tc(ModelDims md, Prefil
 // Same work split as k_pf_attn_tc (one CTA per sequence, block of QT = 128/G queries and kv head;
 // the 128 MMA rows are query * G + head; cache pages of 64 slots), with the roles split across
 // warps so that no block-wide barrier sits in the page loop:
-//   warp 4      TMA producer: the K and V segments of every page, straight from the paged pool
-//               through a 3-D tensor map (128-byte swizzle), into two-deep K and V rings;
+//   warp 4      TMA producer: the block's q rows (bulk copies, staged in the empty rings), then the
+//               K and V segments of every page, straight from the paged pool through a 3-D tensor
+//               map (128-byte swizzle), into K and V rings (three deep for head_dim 128);
 //   warp 5      MMA issuer: S(p) = Q K(p)^T into one of two TMEM buffers (q as bf16 hi + lo terms,
 //               so the scores keep q's float32 precision), then O += P(p-1) V(p-1) with V taken as
 //               an MN-major operand (no transpose);
@@ -605,7 +606,10 @@ struct PfWsShape {
   static constexpr int QCOL = 128 * 128;               // bytes of one atom column of a Q tile
   static constexpr int KV_BYTES = 64 * HD * 2;         // a K (or V) stage: [64 keys][HD]
   static constexpr int KVCOL = 64 * 128;               // bytes of one atom column of a stage
-  static constexpr int NST = 2;                        // ring depth
+  // ring depth: with head_dim 128 a K copy is issued once the S product three pages back has freed
+  // its stage, which covers the copy's latency (two stages left the MMA waiting for K); head_dim 64
+  // keeps two stages so that two CTAs (101 KB each) share an SM and cover it between them
+  static constexpr int NST = HD == 128 ? 3 : 2;
   static constexpr int P_BYTES = 128 * 64 * 2;         // a P buffer [128][64 keys]
   static constexpr int OFF_QHI = 0;
   static constexpr int OFF_QLO = OFF_QHI + Q_BYTES;
@@ -613,13 +617,14 @@ struct PfWsShape {
   static constexpr int OFF_V = OFF_K + NST * KV_BYTES;
   static constexpr int OFF_P = OFF_V + NST * KV_BYTES;
   static constexpr int OFF_BAR = OFF_P + 2 * P_BYTES;
-  static constexpr int NBAR = 4 * NST + 8;
+  static constexpr int NBAR = 4 * NST + 9;
+  static_assert(128 * HD * 4 <= 2 * NST * KV_BYTES, "the float32 Q tile is staged in the K/V rings");
   static constexpr int BYTES = OFF_BAR + NBAR * 8 + 16 + 1024;  // barriers, TMEM slot, alignment slack
   static constexpr uint32_t TMEM_COLS = 256;          // S buffers in columns 0..127, O in 128..128+HD
 };
 
 template <int HD, int G>
-__global__ void __launch_bounds__(PFW_THREADS) k_pf_attn_ws(ModelDims md, PrefillDev p, StepDev s, int r, int j,
+__global__ void __launch_bounds__(PFW_THREADS, HD == 64 ? 2 : 1) k_pf_attn_ws(ModelDims md, PrefillDev p, StepDev s, int r, int j,
                                                              const float* __restrict__ Q, bf16* __restrict__ O,
                                                              const __grid_constant__ CUtensorMap pool_map) {
   using Sh = PfWsShape<HD>;
@@ -638,6 +643,7 @@ __global__ void __launch_bounds__(PFW_THREADS) k_pf_attn_ws(ModelDims md, Prefil
   auto s_free = [&](int b) { return bar(4 * NST + 2 + b); };
   auto p_full = [&](int b) { return bar(4 * NST + 4 + b); };
   auto p_free = [&](int b) { return bar(4 * NST + 6 + b); };
+  const uint32_t q_full = bar(4 * NST + 8);
 
   pdl_wait();
   pdl_trigger();
@@ -675,20 +681,30 @@ __global__ void __launch_bounds__(PFW_THREADS) k_pf_attn_ws(ModelDims md, Prefil
       mbar_init(p_full(b), 4);
       mbar_init(p_free(b), 1);
     }
+    mbar_init(q_full, 1);
     fence_barrier_init();
     prefetch_tensormap(&pool_map);
+    // the block's float32 q rows, staged in the (still unused) K/V rings: the G heads of a query
+    // are contiguous, so one bulk copy per query
+    mbar_arrive_expect_tx(q_full, (uint32_t)(nq * G * HD * 4));
+    for (int qq = 0; qq < nq; ++qq)
+      bulk_g2s(smem_u32(sm + Sh::OFF_K + qq * G * HD * 4), Q + ((size_t)(first + q0 + qq) * md.Hq + kvh * G) * HD,
+               (uint32_t)(G * HD * 4), q_full);
   }
   if (warp == 5) {
     tmem_alloc(smem_u32(tmem_slot), Sh::TMEM_COLS);
     tmem_relinquish();
   }
+  __syncthreads();  // barriers initialised
+  const bool q_ok = __all_sync(0xffffffffu, mbar_wait(q_full, 0, s.err));
   // Q tile: row = query * G + head, as hi and lo bf16 parts (zeros past the block's queries)
+  const float* qstage = reinterpret_cast<const float*>(sm + Sh::OFF_K);
   for (int e = tid; e < 128 * (HD / 8); e += PFW_THREADS) {
     const int qr = e / (HD / 8), c = e % (HD / 8);
-    const int qq = qr / G, gg = qr % G;
+    const int qq = qr / G;
     float x[8];
-    if (qq < nq) {
-      const float4* q4 = reinterpret_cast<const float4*>(Q + ((size_t)(first + q0 + qq) * md.Hq + kvh * G + gg) * HD);
+    if (qq < nq && q_ok) {
+      const float4* q4 = reinterpret_cast<const float4*>(qstage + (size_t)qr * HD);
       const float4 a = q4[2 * c], b = q4[2 * c + 1];
       x[0] = a.x; x[1] = a.y; x[2] = a.z; x[3] = a.w; x[4] = b.x; x[5] = b.y; x[6] = b.z; x[7] = b.w;
     } else {
@@ -762,45 +778,71 @@ __global__ void __launch_bounds__(PFW_THREADS) k_pf_attn_ws(ModelDims md, Prefil
     // ---------------- MMA issuer ----------------
     if (lane == 0) {
       constexpr uint32_t IDS = idesc_bf16_f32(128, 64), IDO = idesc_bf16_f32_bmn(128, HD);
-      auto issue_pv = [&](int q) {  // O += P(q) V(q)
-        const int bq = q & 1, st = q % NST;
-        if (!wait(p_full(bq), (uint32_t)(q >> 1) & 1u) || !wait(v_full(st), (uint32_t)(q / NST) & 1u)) return false;
-        tc_fence_after();
-        const uint32_t pa = smem_u32(sm + Sh::OFF_P + bq * Sh::P_BYTES);
-        const uint32_t vb = smem_u32(sm + Sh::OFF_V + st * Sh::KV_BYTES);
-#pragma unroll
-        for (int k = 0; k < 4; ++k)  // K = 16 keys per MMA: +32 B in P's rows, +2048 B (16 rows) in V
-          tc_mma_f16(tmem + OCOL, smem_desc_sw128(pa) + 2 * k, smem_desc_sw128_mn(vb + 2048u * k, Sh::KVCOL), IDO,
-                     (q > 0 || k > 0) ? 1u : 0u);
-        tc_commit(p_free(bq));
-        tc_commit(v_empty(st));
-        return true;
-      };
-      bool ok = true;
-      for (int pg = 0; pg < npages && ok; ++pg) {
-        const int b = pg & 1, st = pg % NST;
-        if (!wait(k_full(st), (uint32_t)(pg / NST) & 1u)) break;
-        if (pg >= 2 && !wait(s_free(b), (uint32_t)((pg - 2) >> 1) & 1u)) break;
-        tc_fence_after();
-        const uint32_t kb = smem_u32(sm + Sh::OFF_K + st * Sh::KV_BYTES);
-#pragma unroll
-        for (int kc = 0; kc < Sh::ATOMS; ++kc)
-#pragma unroll
-          for (int k = 0; k < 4; ++k) {  // K = 16 per MMA: +32 bytes (encoded +2) inside the atom column
-            const uint64_t db = smem_desc_sw128(kb + kc * Sh::KVCOL) + 2 * k;
+      // every operand descriptor is a base plus a constant step (encoded in 16-byte units), built
+      // once: this thread's instruction count per page is what paces the loop
+      const uint64_t dqh = smem_desc_sw128(smem_u32(sm + Sh::OFF_QHI));
+      const uint64_t dql = smem_desc_sw128(smem_u32(sm + Sh::OFF_QLO));
+      const uint64_t dk0 = smem_desc_sw128(smem_u32(sm + Sh::OFF_K));
+      const uint64_t dp0 = smem_desc_sw128(smem_u32(sm + Sh::OFF_P));
+      const uint64_t dv0 = smem_desc_sw128_mn(smem_u32(sm + Sh::OFF_V), Sh::KVCOL);
+      constexpr uint64_t QCOL_E = Sh::QCOL >> 4, KVCOL_E = Sh::KVCOL >> 4, KV_E = Sh::KV_BYTES >> 4,
+                         P_E = Sh::P_BYTES >> 4, V16_E = 2048 >> 4;
+      // Two streams, each issued as soon as its inputs are there: S(ns) once K(ns) has landed and the
+      // softmax has read the S buffer two pages back, and P V(npv) once P(npv) and V(npv) are in.
+      // S therefore runs ahead of the softmax instead of behind the P V product before it. One time
+      // limit covers the whole loop.
+      int ns = 0, npv = 0;
+      const uint64_t t0 = globaltimer_ns();
+      while (npv < npages) {
+        bool did = false;
+        if (ns < npages) {
+          const int b = ns & 1, st = ns % NST;
+          if (mbar_try_wait(k_full(st), (uint32_t)(ns / NST) & 1u) &&
+              (ns < 2 || mbar_try_wait(s_free(b), (uint32_t)((ns - 2) >> 1) & 1u))) {
+            tc_fence_after();
+            const uint64_t kb = dk0 + st * KV_E;
             const uint32_t d = tmem + 64u * (uint32_t)b;
-            tc_mma_f16(d, smem_desc_sw128(smem_u32(sm + Sh::OFF_QHI + kc * Sh::QCOL)) + 2 * k, db, IDS,
-                       (kc | k) ? 1u : 0u);
-            tc_mma_f16(d, smem_desc_sw128(smem_u32(sm + Sh::OFF_QLO + kc * Sh::QCOL)) + 2 * k, db, IDS, 1u);
+#pragma unroll
+            for (int kc = 0; kc < Sh::ATOMS; ++kc)
+#pragma unroll
+              for (int k = 0; k < 4; ++k) {  // K = 16 per MMA: +32 bytes (encoded +2) inside the atom column
+                const uint64_t db = kb + kc * KVCOL_E + 2 * k;
+                tc_mma_f16(d, dqh + kc * QCOL_E + 2 * k, db, IDS, (kc | k) ? 1u : 0u);
+                tc_mma_f16(d, dql + kc * QCOL_E + 2 * k, db, IDS, 1u);
+              }
+            tc_commit(s_full(b));
+            tc_commit(k_empty(st));
+            ++ns;
+            did = true;
           }
-        tc_commit(s_full(b));
-        tc_commit(k_empty(st));
-        if (pg >= 1) ok = issue_pv(pg - 1);
+        }
+        if (npv < ns) {
+          const int bq = npv & 1, st = npv % NST;
+          if (mbar_try_wait(p_full(bq), (uint32_t)(npv >> 1) & 1u) &&
+              mbar_try_wait(v_full(st), (uint32_t)(npv / NST) & 1u)) {  // O += P(npv) V(npv)
+            tc_fence_after();
+            const uint64_t pa = dp0 + bq * P_E, vb = dv0 + st * KV_E;
+#pragma unroll
+            for (int k = 0; k < 4; ++k)  // K = 16 keys per MMA: +32 B in P's rows, +2048 B (16 rows) in V
+              tc_mma_f16(tmem + OCOL, pa + 2 * k, vb + V16_E * k, IDO, (npv > 0 || k > 0) ? 1u : 0u);
+            tc_commit(p_free(bq));
+            tc_commit(v_empty(st));
+            ++npv;
+            did = true;
+          }
+        }
+        if (!did && (*abort_flag || globaltimer_ns() - t0 > kWaitLimitNs)) {
+          atomicOr(s.err, DEVERR_WAIT);
+          *abort_flag = 1;
+          break;
+        }
       }
-      if (ok) issue_pv(npages - 1);
     }
   } else {
     // ---------------- softmax: thread = MMA row = TMEM lane ----------------
+    // The page's work per thread is short; what bounds it is the length of its dependent chains,
+    // so the row maximum and sum run as four independent partials and no per-key select is taken
+    // (ex2 of -inf is 0 once the reference maximum is finite).
     const int row = warp * 32 + lane;
     const uint32_t t_row = tmem + ((uint32_t)(warp * 32) << 16);
     const int qi = row / G, g = row % G;
@@ -822,12 +864,12 @@ __global__ void __launch_bounds__(PFW_THREADS) k_pf_attn_ws(ModelDims md, Prefil
       __syncwarp();
       if (lane == 0) mbar_arrive(s_free(b));
       const int kb = pg * 64;  // cache slot of column 0
-      float pm = -INFINITY;
+      float pm4[4] = {-INFINITY, -INFINITY, -INFINITY, -INFINITY};
       if (row_ok && kb + 63 <= qslot) {  // every key visible
 #pragma unroll
         for (int c = 0; c < 64; ++c) {
           sc[c] *= scale;
-          pm = fmaxf(pm, sc[c]);
+          pm4[c & 3] = fmaxf(pm4[c & 3], sc[c]);
         }
       } else if (!row_ok || kb > qslot) {  // none visible
 #pragma unroll
@@ -836,9 +878,10 @@ __global__ void __launch_bounds__(PFW_THREADS) k_pf_attn_ws(ModelDims md, Prefil
 #pragma unroll
         for (int c = 0; c < 64; ++c) {
           sc[c] = kb + c <= qslot ? sc[c] * scale : -INFINITY;
-          pm = fmaxf(pm, sc[c]);
+          pm4[c & 3] = fmaxf(pm4[c & 3], sc[c]);
         }
       }
+      const float pm = fmaxf(fmaxf(pm4[0], pm4[1]), fmaxf(pm4[2], pm4[3]));
       // lazy maximum: O is rescaled only when a row's maximum grows by more than 8, after the
       // P V product before has landed (warp-uniform TMEM access)
       const bool grow = pm > m_run + 8.f;
@@ -860,16 +903,16 @@ __global__ void __launch_bounds__(PFW_THREADS) k_pf_attn_ws(ModelDims md, Prefil
         l_run *= cr;
         m_run = pm;
       }
+      const float mref = m_run == -INFINITY ? 0.f : m_run;  // rows with no visible key so far
       uint32_t pk[32];
-      float psum = 0.f;
+      float ps4[4] = {0.f, 0.f, 0.f, 0.f};
 #pragma unroll
       for (int c = 0; c < 64; c += 2) {
-        const float p0 = sc[c] == -INFINITY ? 0.f : ex2_approx(sc[c] - m_run);
-        const float p1 = sc[c + 1] == -INFINITY ? 0.f : ex2_approx(sc[c + 1] - m_run);
-        psum += p0 + p1;
+        const float p0 = ex2_approx(sc[c] - mref), p1 = ex2_approx(sc[c + 1] - mref);
+        ps4[(c >> 1) & 3] += p0 + p1;
         pk[c / 2] = pack_bf16(p0, p1);
       }
-      l_run += psum;
+      l_run += (ps4[0] + ps4[1]) + (ps4[2] + ps4[3]);
       // P buffer b was last read by P V of page pg - 2
       if (pg >= 2 && !wait_w(p_free(b), (uint32_t)((pg - 2) >> 1) & 1u)) { ok = false; break; }
       uint8_t* pb = sm + Sh::OFF_P + b * Sh::P_BYTES;
