@@ -1288,7 +1288,8 @@ static int prefill_batched(tlf_ctx* ctx, int n_seqs, const int* slot_of, const i
         a.row_cslot = ctx->d_pf_row_cslot + (size_t)r * C;
         a.row_pos = ctx->d_pf_row_pos + (size_t)r * C;
         gemm_pf(ctx, ctx->wqkv[j], &ctx->pf_map_X, a, T, st);
-        launch_pf_attn(md, P, sp, r, j, ctx->d_pf_Q, ctx->d_pf_O, C / P.qblock + S + 1, st,
+        // attention blocks of loop r: sum over sequences of ceil(count / qblock) <= T / qblock + S
+        launch_pf_attn(md, P, sp, r, j, ctx->d_pf_Q, ctx->d_pf_O, T / P.qblock + S + 1, st,
                        ctx->has_pool_map && ctx->pf_ws ? &ctx->map_pool : nullptr);
         a = GemmArgs{};
         a.n_dev = n_dev;
