@@ -363,12 +363,14 @@ __device__ __forceinline__ void tmem_ld_acc(uint32_t taddr, int lo_off, float* v
   }
 }
 
-template <int NT>
+// LO: the token operand is two-term (hi + lo planes); a compile-time choice, so the one-plane
+// instantiations (prefill, the LM head) carry none of its code.
+template <int NT, bool LO>
 __global__ void __launch_bounds__(128) k_gemm_tc(const __grid_constant__ CUtensorMap mapW,
                                                  const __grid_constant__ CUtensorMap mapX, GemmArgs a) {
   constexpr int A_BYTES = TC_BM * TC_BK * 2;
-  const bool lo = a.blo > 0;  // two-term token operand
-  const uint32_t TMEM_COLS = (uint32_t)tc_tmem_cols(NT, lo);
+  constexpr bool lo = LO;
+  constexpr uint32_t TMEM_COLS = (uint32_t)tc_tmem_cols(NT, lo);
   const int B_BYTES = tc_b_bytes(NT, lo);
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
@@ -607,16 +609,15 @@ int gemm_tc_stages(int K, int splits, int nt, bool lo) {
 int gemm_tc_smem_bytes(int nt, int stages, bool lo) { return tc_smem_bytes(nt, stages, lo); }
 
 
-template <int NT>
+template <int NT, bool LO>
 static void launch_tc_nt(const CUtensorMap* mapW, const CUtensorMap* mapX, GemmArgs a, cudaStream_t st) {
   static bool attr_set = false;
   if (!attr_set) {
-    const int one = tc_smem_bytes(NT, tc_max_stages(NT, false), false);
-    const int two = tc_smem_bytes(NT, tc_max_stages(NT, true), true);
-    cudaFuncSetAttribute(k_gemm_tc<NT>, cudaFuncAttributeMaxDynamicSharedMemorySize, one > two ? one : two);
+    cudaFuncSetAttribute(k_gemm_tc<NT, LO>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                         tc_smem_bytes(NT, tc_max_stages(NT, LO), LO));
     attr_set = true;
   }
-  a.stages = gemm_tc_stages(a.K, a.splits, NT, a.blo > 0);
+  a.stages = gemm_tc_stages(a.K, a.splits, NT, LO);
   int red_cols = NT;
   if (a.red_window > 0 && a.splits == 1 && a.red_window < NT) {
     // windowed one-split epilogue: with a 2-stage ring two CTAs share an SM, so one CTA's
@@ -626,16 +627,16 @@ static void launch_tc_nt(const CUtensorMap* mapW, const CUtensorMap* mapX, GemmA
   } else {
     a.red_window = 0;
   }
-  const int smem = tc_smem_bytes(NT, a.stages, a.blo > 0, red_cols);
+  const int smem = tc_smem_bytes(NT, a.stages, LO, red_cols);
   dim3 grid((a.N + TC_BM - 1) / TC_BM, a.splits, a.tok_tiles > 0 ? a.tok_tiles : 1);
   if (a.epi < EPI_CL_RESID) {
-    launch_k(k_gemm_tc<NT>, grid, 128, smem, st, *mapW, *mapX, a);
+    launch_k(k_gemm_tc<NT, LO>, grid, 128, smem, st, *mapW, *mapX, a);
     return;
   }
   // cluster epilogue: the splits of one tile form a (1, splits, 1) cluster
   static bool nonportable = false;
   if (a.splits > 8 && !nonportable) {
-    cudaFuncSetAttribute(k_gemm_tc<NT>, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
+    cudaFuncSetAttribute(k_gemm_tc<NT, LO>, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
     nonportable = true;
   }
   cudaLaunchConfig_t cfg = {};
@@ -652,18 +653,25 @@ static void launch_tc_nt(const CUtensorMap* mapW, const CUtensorMap* mapX, GemmA
   attr[1].val.programmaticStreamSerializationAllowed = 1;
   cfg.attrs = attr;
   cfg.numAttrs = g_use_pdl ? 2 : 1;
-  cudaLaunchKernelEx(&cfg, k_gemm_tc<NT>, *mapW, *mapX, a);
+  cudaLaunchKernelEx(&cfg, k_gemm_tc<NT, LO>, *mapW, *mapX, a);
+}
+
+template <bool LO>
+static void launch_tc(const CUtensorMap* mapW, const CUtensorMap* mapX, int nt_max, const GemmArgs& a,
+                      cudaStream_t st) {
+  switch (nt_max) {
+    case 16: launch_tc_nt<16, LO>(mapW, mapX, a, st); break;
+    case 32: launch_tc_nt<32, LO>(mapW, mapX, a, st); break;
+    case 64: launch_tc_nt<64, LO>(mapW, mapX, a, st); break;
+    case 128: launch_tc_nt<128, LO>(mapW, mapX, a, st); break;
+    default: launch_tc_nt<256, LO>(mapW, mapX, a, st); break;
+  }
 }
 
 void launch_gemm_tc(const CUtensorMap* mapW, const CUtensorMap* mapX, int nt_max, const GemmArgs& a,
                     cudaStream_t st) {
-  switch (nt_max) {
-    case 16: launch_tc_nt<16>(mapW, mapX, a, st); break;
-    case 32: launch_tc_nt<32>(mapW, mapX, a, st); break;
-    case 64: launch_tc_nt<64>(mapW, mapX, a, st); break;
-    case 128: launch_tc_nt<128>(mapW, mapX, a, st); break;
-    default: launch_tc_nt<256>(mapW, mapX, a, st); break;
-  }
+  if (a.blo > 0) launch_tc<true>(mapW, mapX, nt_max, a, st);
+  else launch_tc<false>(mapW, mapX, nt_max, a, st);
 }
 
 // ----------------------------------------------------------------------------
