@@ -118,14 +118,17 @@ __global__ void __launch_bounds__(ATT_THREADS) k_attn_decode(ModelDims md, StepD
   }
   __syncthreads();
 
-  // (token, kv head, page) of flat page p
+  // (token, kv head, page) of flat page p: the largest k with pbase[k] <= p, found by the warp
+  // with independent loads (32 entries of pbase a round) and a ballot
   auto locate = [&](int p, int& k, int& h, int& g) {
-    int lo = 0, hi = n_r;  // largest k with pbase[k] <= p
-    while (hi - lo > 1) {
-      const int mid = (lo + hi) >> 1;
-      if (pbase[mid] <= p) lo = mid; else hi = mid;
+    int kk = 0;
+    for (int b = 0; b < n_r; b += 32) {
+      const int i = b + lane;
+      const unsigned le = __ballot_sync(0xffffffffu, i < n_r && pbase[i] <= p);
+      if (le) kk = b + 31 - __clz((int)le);
+      if (le != 0xffffffffu) break;  // pbase is non-decreasing: no later entry is <= p
     }
-    k = lo;
+    k = kk;
     const int off = p - pbase[k], np = pages_of(k);
     h = off / np;
     g = off % np;
@@ -133,10 +136,10 @@ __global__ void __launch_bounds__(ATT_THREADS) k_attn_decode(ModelDims md, StepD
 
   if (warp == ATT_WARPS) {
     // ---------------- producer warp ----------------
+    int k, h, g;
+    locate(p0, k, h, g);  // the whole warp (ballot)
     if (lane == 0) {
       const uint64_t kv_policy = l2_policy_evict_first();  // pages are read once per launch
-      int k, h, g;
-      locate(p0, k, h, g);
       int slot = s.slots[s.idx[r * maxB + k]];
       int L = nkeys[k];
       for (int p = p0; p < p1; ++p) {

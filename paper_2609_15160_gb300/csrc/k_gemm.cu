@@ -42,6 +42,8 @@
 // Other epilogues (SIMT path, LM head): split-K partial sums to a buffer
 // consumed by k_rope_append / k_swiglu, atomic residual add + scatter, or a
 // plain float32 store (logits).
+#include <type_traits>
+
 #include "tlf_internal.cuh"
 
 namespace tlf {
@@ -192,33 +194,44 @@ __device__ void cluster_epilogue(const GemmArgs& a, float* red, int4* ci, const 
     const bool fin = col < a.N;
     const float gain = fin ? a.gain[col] : 0.f;
     const int warp = tid >> 5, lane = tid & 31;
-    // column c (uniform over the CTA): h is its residual value before the update
-    auto finish = [&](int c, float h, float sm) {
+    // column c (uniform over the CTA): h is its residual value before the update; returns the
+    // square of the updated value (the next norm's share of this feature)
+    auto update = [&](int c, float h, float sm) {
       const int4 e = ci[c];
       if (fin && e.w >= 0) {  // the only writer of this element
         const float g = a.alpha.mod ? a.alpha.mod[e.x + col] : 1.f;
         h += g * sm;
         a.resid[(size_t)e.w * a.ldr + col] = h;
       }
-      if (e.z >= 0) {
-        if (fin) {
-          const float gm = a.gamma.mod ? 1.f + a.gamma.mod[e.y + col] : 1.f;
-          const float y = h * gain * gm;
-          const bf16 yh = __float2bfloat16_rn(y);
-          a.xn[(size_t)e.z * a.N + col] = yh;
-          if (a.xn_lo) a.xn_lo[(size_t)e.z * a.N + col] = __float2bfloat16_rn(y - __bfloat162float(yh));
-        }
-        const float t = warp_sum(h * h);
-        if (lane == 0) ssp[warp * NT + c] = t;
+      if (e.z >= 0 && fin) {
+        const float gm = a.gamma.mod ? 1.f + a.gamma.mod[e.y + col] : 1.f;
+        const float y = h * gain * gm;
+        const bf16 yh = __float2bfloat16_rn(y);
+        a.xn[(size_t)e.z * a.N + col] = yh;
+        if (a.xn_lo) a.xn_lo[(size_t)e.z * a.N + col] = __float2bfloat16_rn(y - __bfloat162float(yh));
       }
+      return h * h;
+    };
+    // the warp sums of Q columns' squares, their shuffle chains interleaved
+    auto sums = [&](int c, float* t, auto qn) {
+      constexpr int Q = decltype(qn)::value;
+#pragma unroll
+      for (int o = 16; o > 0; o >>= 1)
+#pragma unroll
+        for (int q = 0; q < Q; ++q) t[q] += __shfl_xor_sync(0xffffffffu, t[q], o);
+      if (lane == 0)
+#pragma unroll
+        for (int q = 0; q < Q; ++q)
+          if (c + q < c1 && ci[c + q].z >= 0) ssp[warp * NT + c + q] = t[q];
     };
     if (c1 - c0 <= HPRE) {
       float sm[HPRE];
 #pragma unroll
       for (int q = 0; q < HPRE; q += 4) cluster_sum4(pb, red, 0, S, tid, c0 + q, c1, sm + q);
+      float t[HPRE];
 #pragma unroll
-      for (int q = 0; q < HPRE; ++q)
-        if (c0 + q < c1) finish(c0 + q, hpre[q], sm[q]);
+      for (int q = 0; q < HPRE; ++q) t[q] = (c0 + q < c1) ? update(c0 + q, hpre[q], sm[q]) : 0.f;
+      sums(c0, t, std::integral_constant<int, HPRE>{});
     } else {
       for (int c = c0; c < c1; c += 4) {
         float hv[4];
@@ -229,9 +242,10 @@ __device__ void cluster_epilogue(const GemmArgs& a, float* red, int4* ci, const 
         }
         float sm[4];
         cluster_sum4(pb, red, 0, S, tid, c, c1, sm);
+        float t[4];
 #pragma unroll
-        for (int q = 0; q < 4; ++q)
-          if (c + q < c1) finish(c + q, hv[q], sm[q]);
+        for (int q = 0; q < 4; ++q) t[q] = (c + q < c1) ? update(c + q, hv[q], sm[q]) : 0.f;
+        sums(c, t, std::integral_constant<int, 4>{});
       }
     }
     __syncthreads();
@@ -352,15 +366,15 @@ __device__ void cluster_epilogue(const GemmArgs& a, float* red, int4* ci, const 
   }
 }
 
-// 16 accumulator columns; with a two-term operand (lo_off > 0) plus the lo half lo_off columns on.
+// 16 accumulator columns; with a two-term operand (lo_off > 0) plus the lo half lo_off columns on
+// (both loads in flight before one wait).
 __device__ __forceinline__ void tmem_ld_acc(uint32_t taddr, int lo_off, float* v) {
-  tmem_ld_16(taddr, v);
-  if (lo_off > 0) {
-    float w[16];
-    tmem_ld_16(taddr + (uint32_t)lo_off, w);
+  uint32_t r[16], w[16];
+  tmem_ld_16_issue(taddr, r);
+  if (lo_off > 0) tmem_ld_16_issue(taddr + (uint32_t)lo_off, w);
+  tmem_ld_wait();
 #pragma unroll
-    for (int i = 0; i < 16; ++i) v[i] += w[i];
-  }
+  for (int i = 0; i < 16; ++i) v[i] = lo_off > 0 ? __uint_as_float(r[i]) + __uint_as_float(w[i]) : __uint_as_float(r[i]);
 }
 
 // LO: the token operand is two-term (hi + lo planes); a compile-time choice, so the one-plane
