@@ -374,12 +374,8 @@ __global__ void __launch_bounds__(ATT_THREADS) k_attn_decode(ModelDims md, StepD
 template <typename T, int HD, int G, bool MASKED>
 static void attn_launch_v(const ModelDims& md, const StepDev& s, int r, int j, const float* Q, float* part, void* O,
                           int* cnt, int grid, cudaStream_t st, bool o_lo) {
-  static bool attr = false;
   constexpr int smem = attn_smem_bytes<T, HD, G, MASKED>();
-  if (!attr) {
-    cudaFuncSetAttribute(k_attn_decode<T, HD, G, MASKED>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
-    attr = true;
-  }
+  (void)ensure_kernel_attrs((const void*)k_attn_decode<T, HD, G, MASKED>, smem);  // a failure shows at launch
   launch_k(k_attn_decode<T, HD, G, MASKED>, grid, ATT_THREADS, smem, st, md, s, r, j, Q, part, (T*)O, cnt, o_lo);
 }
 

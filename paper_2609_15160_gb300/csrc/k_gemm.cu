@@ -625,12 +625,8 @@ int gemm_tc_smem_bytes(int nt, int stages, bool lo) { return tc_smem_bytes(nt, s
 
 template <int NT, bool LO>
 static void launch_tc_nt(const CUtensorMap* mapW, const CUtensorMap* mapX, GemmArgs a, cudaStream_t st) {
-  static bool attr_set = false;
-  if (!attr_set) {
-    cudaFuncSetAttribute(k_gemm_tc<NT, LO>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                         tc_smem_bytes(NT, tc_max_stages(NT, LO), LO));
-    attr_set = true;
-  }
+  // (a failure shows at launch)
+  (void)ensure_kernel_attrs((const void*)k_gemm_tc<NT, LO>, tc_smem_bytes(NT, tc_max_stages(NT, LO), LO));
   a.stages = gemm_tc_stages(a.K, a.splits, NT, LO);
   int red_cols = NT;
   if (a.red_window > 0 && a.splits == 1 && a.red_window < NT) {
@@ -648,11 +644,8 @@ static void launch_tc_nt(const CUtensorMap* mapW, const CUtensorMap* mapX, GemmA
     return;
   }
   // cluster epilogue: the splits of one tile form a (1, splits, 1) cluster
-  static bool nonportable = false;
-  if (a.splits > 8 && !nonportable) {
-    cudaFuncSetAttribute(k_gemm_tc<NT, LO>, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
-    nonportable = true;
-  }
+  if (a.splits > 8)
+    (void)ensure_kernel_attrs((const void*)k_gemm_tc<NT, LO>, tc_smem_bytes(NT, tc_max_stages(NT, LO), LO), true);
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = grid;
   cfg.blockDim = dim3(128);

@@ -959,12 +959,8 @@ __global__ void k_pf_len(ModelDims md, PrefillDev p) {
 template <typename T, int HD, int G>
 static void pf_attn_launch(const ModelDims& md, const PrefillDev& p, const StepDev& s, int r, int j, const float* Q,
                            void* O, int tiles_bound, cudaStream_t st) {
-  static bool attr = false;
   constexpr int smem = (PF_QB * G * HD + HD * 65 + 64 * HD + PF_WARPS * (PF_QB / PF_WARPS) * G * 64) * 4;
-  if (!attr) {
-    cudaFuncSetAttribute(k_pf_attn<T, HD, G>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
-    attr = true;
-  }
+  (void)ensure_kernel_attrs((const void*)k_pf_attn<T, HD, G>, smem);  // a failure shows at launch
   launch_k(k_pf_attn<T, HD, G>, dim3(tiles_bound, md.Hkv), 32 * PF_WARPS, smem, st, md, p, s, r, j, Q, (T*)O);
 }
 
@@ -975,24 +971,16 @@ void launch_pf_plan(const ModelDims& md, const PrefillDev& p, cudaStream_t st) {
 template <int HD, int G>
 static void pf_attn_tc_launch(const ModelDims& md, const PrefillDev& p, const StepDev& s, int r, int j,
                               const float* Q, void* O, int tiles_bound, cudaStream_t st) {
-  static bool attr = false;
   constexpr int smem = PfTcShape<HD>::BYTES;
-  if (!attr) {
-    cudaFuncSetAttribute(k_pf_attn_tc<HD, G>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
-    attr = true;
-  }
+  (void)ensure_kernel_attrs((const void*)k_pf_attn_tc<HD, G>, smem);  // a failure shows at launch
   launch_k(k_pf_attn_tc<HD, G>, dim3(tiles_bound, md.Hkv), PFT_THREADS, smem, st, md, p, s, r, j, Q, (bf16*)O);
 }
 
 template <int HD, int G>
 static void pf_attn_ws_launch(const ModelDims& md, const PrefillDev& p, const StepDev& s, int r, int j,
                               const float* Q, void* O, int tiles_bound, cudaStream_t st, const CUtensorMap* pool_map) {
-  static bool attr = false;
   constexpr int smem = PfWsShape<HD>::BYTES;
-  if (!attr) {
-    cudaFuncSetAttribute(k_pf_attn_ws<HD, G>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
-    attr = true;
-  }
+  (void)ensure_kernel_attrs((const void*)k_pf_attn_ws<HD, G>, smem);  // a failure shows at launch
   launch_k(k_pf_attn_ws<HD, G>, dim3(tiles_bound * md.Hkv), PFW_THREADS, smem, st, md, p, s, r, j, Q, (bf16*)O,
            *pool_map);
 }

@@ -372,14 +372,9 @@ void launch_router(const ModelDims& md, const StepDev& s, int B, const void* emb
                    const void* router_w1, const float* router_b1) {
   if (md.router_hidden > 0) {
     const size_t smem = (size_t)(md.d + md.router_hidden) * 4;
-    static bool attr[2] = {false, false};
-    if (!attr[md.dtype]) {
-      if (md.dtype == 1)
-        cudaFuncSetAttribute(k_router_mlp<bf16>, cudaFuncAttributeMaxDynamicSharedMemorySize, 65536);
-      else
-        cudaFuncSetAttribute(k_router_mlp<float>, cudaFuncAttributeMaxDynamicSharedMemorySize, 65536);
-      attr[md.dtype] = true;
-    }
+    // (a failure shows at launch)
+    (void)ensure_kernel_attrs(md.dtype == 1 ? (const void*)k_router_mlp<bf16> : (const void*)k_router_mlp<float>,
+                              65536);
     if (md.dtype == 1)
       launch_k(k_router_mlp<bf16>, B, 256, smem, st, md, s, B, (const bf16*)emb, (const bf16*)router_w1, router_b1,
                (const bf16*)router_w, router_b, upd, n_upd);

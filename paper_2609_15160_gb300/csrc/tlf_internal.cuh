@@ -572,6 +572,12 @@ void launch_rope_append(const ModelDims& md, const StepDev& s, int r, int j, con
 // max_batch, the two-term operand of the output projection
 void launch_attn_decode(const ModelDims& md, const StepDev& s, int r, int j, const float* Q, float* part, void* O,
                         int* cnt, int grid, cudaStream_t st, bool o_lo = false);
+// Id of the calling thread's current CUDA context (unique for the life of the process); false when
+// no context is current yet or the driver entry points are unavailable.
+bool current_context_id(unsigned long long* id);
+// A kernel's dynamic shared-memory limit (and, if asked, non-portable cluster sizes), set once per
+// (kernel, CUDA context).
+cudaError_t ensure_kernel_attrs(const void* func, int max_dyn_smem, bool nonportable_cluster = false);
 int attn_decode_grid(const ModelDims& md, int num_sms);
 size_t attn_partial_floats(const ModelDims& md, int grid);
 

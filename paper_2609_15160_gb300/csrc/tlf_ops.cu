@@ -6,12 +6,73 @@
 // lengths, the plan kernel cuts every (row, kv head) key range into chunks,
 // k_attn_decode streams the pages and k_attn_combine merges the chunk
 // partials. The scratch holds the plan and the partials.
+#include <cudaTypedefs.h>
+
 #include <atomic>
+#include <mutex>
+#include <vector>
 
 #include "tlf.h"
 #include "tlf_internal.cuh"
 
 namespace tlf {
+
+// Id of the calling thread's current CUDA context (unique for the life of the process);
+// false when no context is current yet or the driver entry points are unavailable.
+bool current_context_id(unsigned long long* id) {
+  static std::atomic<PFN_cuCtxGetCurrent_v4000> get_current{nullptr};
+  static std::atomic<PFN_cuCtxGetId_v12000> get_id{nullptr};
+  if (!get_current.load() || !get_id.load()) {
+    void* p = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuCtxGetCurrent", &p, 4000, cudaEnableDefault, &q) != cudaSuccess ||
+        q != cudaDriverEntryPointSuccess || !p)
+      return false;
+    get_current.store(reinterpret_cast<PFN_cuCtxGetCurrent_v4000>(p));
+    p = nullptr;
+    if (cudaGetDriverEntryPointByVersion("cuCtxGetId", &p, 12000, cudaEnableDefault, &q) != cudaSuccess ||
+        q != cudaDriverEntryPointSuccess || !p)
+      return false;
+    get_id.store(reinterpret_cast<PFN_cuCtxGetId_v12000>(p));
+  }
+  CUcontext c = nullptr;
+  if (get_current.load()(&c) != CUDA_SUCCESS || !c) return false;
+  return get_id.load()(c, id) == CUDA_SUCCESS;
+}
+
+// Kernel attributes belong to a CUDA context: a device reset, or the same kernel on another
+// device, needs them set again. Each (kernel, context) pair is set once; without a context id
+// the attributes are set on every call.
+cudaError_t ensure_kernel_attrs(const void* func, int max_dyn_smem, bool nonportable_cluster) {
+  struct Entry {
+    const void* func;
+    unsigned long long ctx;
+    int smem;
+    bool nonportable;
+  };
+  static std::mutex mu;
+  static std::vector<Entry> done;
+  unsigned long long ctx = 0;
+  const bool have = current_context_id(&ctx);
+  std::lock_guard<std::mutex> lock(mu);
+  Entry* hit = nullptr;
+  if (have)
+    for (Entry& e : done)
+      if (e.func == func && e.ctx == ctx) hit = &e;
+  if (hit && hit->smem >= max_dyn_smem && (hit->nonportable || !nonportable_cluster)) return cudaSuccess;
+  cudaError_t r = cudaFuncSetAttribute(func, cudaFuncAttributeMaxDynamicSharedMemorySize, max_dyn_smem);
+  if (r == cudaSuccess && nonportable_cluster)
+    r = cudaFuncSetAttribute(func, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
+  if (r == cudaSuccess && have) {
+    if (hit) {
+      hit->smem = max_dyn_smem;
+      hit->nonportable = hit->nonportable || nonportable_cluster;
+    } else {
+      done.push_back({func, ctx, max_dyn_smem, nonportable_cluster});
+    }
+  }
+  return r;
+}
 
 __global__ void k_attn_prep(int n, const int* __restrict__ lens, int max_keys, int* m, int* slots, int* len,
                             uint32_t* err) {

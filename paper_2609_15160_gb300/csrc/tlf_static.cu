@@ -10,8 +10,6 @@
 // torn down and re-created (cudaDeviceReset, for one) loads the module again,
 // possibly elsewhere, and gets a new id, so the next call looks again instead
 // of handing the kernels a stale address.
-#include <cudaTypedefs.h>
-
 #include <atomic>
 #include <cstdio>
 #include <mutex>
@@ -32,29 +30,6 @@ struct ScratchEntry {
 };
 ScratchEntry g_scratch[kMaxDevices];
 
-// Id of the calling thread's current CUDA context (unique for the life of the process);
-// false when no context is current yet or the driver entry points are unavailable.
-bool current_context_id(unsigned long long* id) {
-  static std::atomic<PFN_cuCtxGetCurrent_v4000> get_current{nullptr};
-  static std::atomic<PFN_cuCtxGetId_v12000> get_id{nullptr};
-  if (!get_current.load() || !get_id.load()) {
-    void* p = nullptr;
-    cudaDriverEntryPointQueryResult q;
-    if (cudaGetDriverEntryPointByVersion("cuCtxGetCurrent", &p, 4000, cudaEnableDefault, &q) != cudaSuccess ||
-        q != cudaDriverEntryPointSuccess || !p)
-      return false;
-    get_current.store(reinterpret_cast<PFN_cuCtxGetCurrent_v4000>(p));
-    p = nullptr;
-    if (cudaGetDriverEntryPointByVersion("cuCtxGetId", &p, 12000, cudaEnableDefault, &q) != cudaSuccess ||
-        q != cudaDriverEntryPointSuccess || !p)
-      return false;
-    get_id.store(reinterpret_cast<PFN_cuCtxGetId_v12000>(p));
-  }
-  CUcontext c = nullptr;
-  if (get_current.load()(&c) != CUDA_SUCCESS || !c) return false;
-  return get_id.load()(c, id) == CUDA_SUCCESS;
-}
-
 // Device address of g_static_scratch in the current device's current context (looked up
 // once per device and context).
 int static_scratch_address(void** out) {
@@ -65,14 +40,14 @@ int static_scratch_address(void** out) {
   std::lock_guard<std::mutex> lock(g_scratch_mu);
   ScratchEntry& ent = g_scratch[dev];
   unsigned long long id = 0;
-  const bool have_id = current_context_id(&id);
+  const bool have_id = tlf::current_context_id(&id);
   if (!have_id || !ent.addr || ent.ctx_id != id) {
     void* p = nullptr;
     e = cudaGetSymbolAddress(&p, g_static_scratch);  // makes the runtime's context current if none was
     if (e != cudaSuccess || !p)
       return tlf::set_thread_error(TLF_ERR_CUDA, e != cudaSuccess ? cudaGetErrorString(e)
                                                                   : "cudaGetSymbolAddress returned NULL");
-    if (!current_context_id(&id))
+    if (!tlf::current_context_id(&id))
       return tlf::set_thread_error(TLF_ERR_CUDA, "no current CUDA context after the symbol lookup");
     ent.ctx_id = id;
     ent.addr = p;
