@@ -1149,7 +1149,9 @@ static void gemm_pf(tlf_ctx* ctx, const DeviceMat& W, const CUtensorMap* xmap, G
   const long long tiles = (long long)((W.N + 127) / 128) * ((rows + 255) / 256);
   a.red_window = tiles > ctx->num_sms ? 128 : 0;
   a.max_rows = ctx->pf_C;
-  a.tok_tiles = ctx->pf_C / 256;
+  // token tiles of the chunk's rows (every loop's rows are among them), not of its capacity: a short
+  // prompt would otherwise launch a grid of CTAs that only wait for the kernel before and exit
+  a.tok_tiles = (rows + 255) / 256;
   launch_gemm_tc(&W.map, xmap, 256, a, st);
 }
 
@@ -1273,7 +1275,8 @@ static int prefill_batched(tlf_ctx* ctx, int n_seqs, const int* slot_of, const i
       const int* n_dev = ctx->d_pf_n + r;
       const int* idx_r = ctx->d_pf_idx + (size_t)r * C;
       for (int j = 0; j < J; ++j) {
-        launch_norm_rows(md.dtype, ctx->d_pf_H, md.d, idx_r, n_dev, 0, C, ctx->d_attn_norm + (size_t)j * md.d, md.d,
+        // one CTA per row of the chunk's T tokens (an upper bound on the loop's rows)
+        launch_norm_rows(md.dtype, ctx->d_pf_H, md.d, idx_r, n_dev, 0, T, ctx->d_attn_norm + (size_t)j * md.d, md.d,
                          md.eps, ctx->d_pf_X, md.d, st, cond_args(ctx, ctx->d_pf_m, r, j, 2));
         GemmArgs a{};
         a.n_dev = n_dev;
@@ -1299,7 +1302,7 @@ static int prefill_batched(tlf_ctx* ctx, int n_seqs, const int* slot_of, const i
         a.idx = idx_r;
         a.alpha = cond_args(ctx, ctx->d_pf_m, r, j, 0);
         gemm_pf(ctx, ctx->wo[j], &ctx->pf_map_O, a, T, st);
-        launch_norm_rows(md.dtype, ctx->d_pf_H, md.d, idx_r, n_dev, 0, C, ctx->d_mlp_norm + (size_t)j * md.d, md.d,
+        launch_norm_rows(md.dtype, ctx->d_pf_H, md.d, idx_r, n_dev, 0, T, ctx->d_mlp_norm + (size_t)j * md.d, md.d,
                          md.eps, ctx->d_pf_X, md.d, st, cond_args(ctx, ctx->d_pf_m, r, j, 3));
         a = GemmArgs{};
         a.n_dev = n_dev;
