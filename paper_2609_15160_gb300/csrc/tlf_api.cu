@@ -1143,15 +1143,23 @@ static void gemm_pf(tlf_ctx* ctx, const DeviceMat& W, const CUtensorMap* xmap, G
   a.K = W.K;
   a.err = ctx->d_err;
   a.splits = 1;
+  const int ntiles = (W.N + 127) / 128, ttiles = (rows + 255) / 256;
+  // A chunk of one token tile (a short prompt) would stream the weights through one CTA per
+  // 128-row tile: K is split over a cluster instead (up to 8 CTAs, at least two k-tiles each), as
+  // in the decode step, while tiles x splits still fit one CTA per SM.
+  if (ttiles == 1 && a.epi >= EPI_CL_RESID) {
+    const int nkb = (W.K + 63) / 64;
+    while (a.splits < 8 && (long long)ntiles * a.splits * 2 <= ctx->num_sms && nkb >= 4 * a.splits) a.splits *= 2;
+  }
   // Stage 128 of the 256 token columns at a time (2-stage ring): two CTAs share an SM, so one
   // CTA's epilogue overlaps the other's main loop. Only worth it when the grid has more tiles
   // than SMs; a smaller grid keeps one CTA per SM and the deeper ring.
-  const long long tiles = (long long)((W.N + 127) / 128) * ((rows + 255) / 256);
-  a.red_window = tiles > ctx->num_sms ? 128 : 0;
+  const long long tiles = (long long)ntiles * ttiles;
+  a.red_window = (a.splits == 1 && tiles > ctx->num_sms) ? 128 : 0;
   a.max_rows = ctx->pf_C;
   // token tiles of the chunk's rows (every loop's rows are among them), not of its capacity: a short
   // prompt would otherwise launch a grid of CTAs that only wait for the kernel before and exit
-  a.tok_tiles = (rows + 255) / 256;
+  a.tok_tiles = ttiles;
   launch_gemm_tc(&W.map, xmap, 256, a, st);
 }
 
