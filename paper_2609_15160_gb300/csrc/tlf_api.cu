@@ -1144,12 +1144,13 @@ static void gemm_pf(tlf_ctx* ctx, const DeviceMat& W, const CUtensorMap* xmap, G
   a.err = ctx->d_err;
   a.splits = 1;
   const int ntiles = (W.N + 127) / 128, ttiles = (rows + 255) / 256;
-  // A chunk of one token tile (a short prompt) would stream the weights through one CTA per
-  // 128-row tile: K is split over a cluster instead (up to 8 CTAs, at least two k-tiles each), as
-  // in the decode step, while tiles x splits still fit one CTA per SM.
-  if (ttiles == 1 && a.epi >= EPI_CL_RESID) {
+  // A chunk of few token tiles (a short prompt) would stream the weights through few CTAs, one per
+  // (128-row tile, token tile): K is split over a cluster instead (up to 8 CTAs, at least two k-tiles
+  // each), as in the decode step, while the tiles x splits still fit one CTA per SM.
+  if (a.epi >= EPI_CL_RESID) {
     const int nkb = (W.K + 63) / 64;
-    while (a.splits < 8 && (long long)ntiles * a.splits * 2 <= ctx->num_sms && nkb >= 4 * a.splits) a.splits *= 2;
+    while (a.splits < 8 && (long long)ntiles * ttiles * a.splits * 2 <= ctx->num_sms && nkb >= 4 * a.splits)
+      a.splits *= 2;
   }
   // Stage 128 of the 256 token columns at a time (2-stage ring): two CTAs share an SM, so one
   // CTA's epilogue overlaps the other's main loop. Only worth it when the grid has more tiles
