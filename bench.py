@@ -197,7 +197,10 @@ def run_reference(args):
     line = {"impl": "reference", "metric": "decode_tokens_per_s", "value": value, "unit": "tokens/s",
             "n_gpus": ws, "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1e3 * sec_per_tok,
             "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
-            "config": {"workload": DESCR[cfg], **synth.describe(wl)},
+            # the same workload keys as the timed arm's line, then the model description
+            "config": {**synth.describe(wl), "workload": DESCR[cfg], "name": cfg, "batch_per_gpu": wl.batch,
+                       "context": int(wl.prompt_len[1]),
+                       "parallelism": f"replicas x{ws} (rank 0 times the oracle; the others exit)"},
             "cpu_baseline": {"value": value, "unit": "tokens/s", "cores": cores, "kind": "oracle",
                              "sample": f"1 sequence at context {d['context']}, 1 decode token per step"},
             "e2e": {"value": value, "unit": "tokens/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}

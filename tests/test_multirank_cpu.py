@@ -70,4 +70,6 @@ def test_reference_arm_under_torchrun():
     assert len(lines) == 1, r.stdout
     d = json.loads(lines[0])
     assert d["impl"] == "reference" and d["n_gpus"] == 2 and d["steps"] == 2 and d["warmup"] == 3
+    # the workload is named as in the timed arm's line
+    assert d["config"]["name"] == "c1" and d["config"]["workload"] != "c1"
     assert d["value"] > 0 and d["e2e"]["h2d_bytes_per_step"] == 0 and d["cpu_baseline"]["kind"] == "oracle"
