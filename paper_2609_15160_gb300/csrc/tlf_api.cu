@@ -137,6 +137,7 @@ struct tlf_ctx {
       *d_pf_row_pos = nullptr, *d_pf_first = nullptr, *d_pf_cnt = nullptr, *d_pf_s0 = nullptr,
       *d_pf_tile_base = nullptr;
   int* h_pf_m = nullptr;
+  int* h_pf_nr = nullptr;  // [M] rows of every loop of the current prefill chunk
   float pf_last_ms = 0.f;
 
   // profiling
@@ -623,6 +624,7 @@ extern "C" void tlf_destroy(tlf_ctx* ctx) {
     f(ctx->d_pf_row_pos); f(ctx->d_pf_first); f(ctx->d_pf_cnt); f(ctx->d_pf_s0); f(ctx->d_pf_tile_base);
     if (ctx->h_pf_in) cudaFreeHost(ctx->h_pf_in);
     if (ctx->h_pf_m) cudaFreeHost(ctx->h_pf_m);
+    if (ctx->h_pf_nr) cudaFreeHost(ctx->h_pf_nr);
     if (ctx->cap_stream) cudaStreamDestroy(ctx->cap_stream);
   }
   delete ctx;
@@ -1108,6 +1110,7 @@ static int ensure_prefill_buffers(tlf_ctx* ctx) {
   if ((rc = dev_alloc(ctx, &ctx->d_pf_in, ctx->pf_in_ints * 4, "prefill inputs"))) return rc;
   CK(ctx, cudaMallocHost((void**)&ctx->h_pf_in, ctx->pf_in_ints * 4));
   CK(ctx, cudaMallocHost((void**)&ctx->h_pf_m, (size_t)C * 4));
+  CK(ctx, cudaMallocHost((void**)&ctx->h_pf_nr, (size_t)M * 4));
   if ((rc = dev_alloc(ctx, &ctx->d_pf_m, (size_t)C * 4, "prefill m"))) return rc;
   if ((rc = dev_alloc(ctx, &ctx->d_pf_margin, (size_t)C * 4, "prefill margin"))) return rc;
   if ((rc = dev_alloc(ctx, &ctx->d_pf_H, (size_t)C * d * 4, "prefill H"))) return rc;
@@ -1274,6 +1277,15 @@ static int prefill_batched(tlf_ctx* ctx, int n_seqs, const int* slot_of, const i
     P.qblock = pf_attn_qblock(md);
     P.len = ctx->d_len;
     launch_pf_plan(md, P, st);
+    // For a chunk of more than one 256-token tile, the rows of every loop come to the host: each
+    // loop's grids follow them (deeper loops hold fewer of the chunk's tokens, so their grids shrink
+    // and their GEMMs may split K), and a loop that no token reaches launches nothing. A chunk of one
+    // tile has nothing to shrink and skips the wait.
+    const bool per_loop_rows = T > 256;
+    if (per_loop_rows) {
+      CK(ctx, cudaMemcpyAsync(ctx->h_pf_nr, ctx->d_pf_n, (size_t)M * 4, cudaMemcpyDeviceToHost, st));
+      CK(ctx, cudaStreamSynchronize(st));
+    }
     StepDev sp{};
     sp.page_table = ctx->d_page_table;
     sp.pool = ctx->d_pool;
@@ -1283,9 +1295,12 @@ static int prefill_batched(tlf_ctx* ctx, int n_seqs, const int* slot_of, const i
     for (int r = 0; r < M; ++r) {
       const int* n_dev = ctx->d_pf_n + r;
       const int* idx_r = ctx->d_pf_idx + (size_t)r * C;
+      // rows of loop r (the kernels read the count itself from n_dev)
+      const int nr = per_loop_rows ? std::min(std::max(ctx->h_pf_nr[r], 0), T) : T;
+      if (nr == 0) continue;
       for (int j = 0; j < J; ++j) {
-        // one CTA per row of the chunk's T tokens (an upper bound on the loop's rows)
-        launch_norm_rows(md.dtype, ctx->d_pf_H, md.d, idx_r, n_dev, 0, T, ctx->d_attn_norm + (size_t)j * md.d, md.d,
+        // one CTA per row of the loop
+        launch_norm_rows(md.dtype, ctx->d_pf_H, md.d, idx_r, n_dev, 0, nr, ctx->d_attn_norm + (size_t)j * md.d, md.d,
                          md.eps, ctx->d_pf_X, md.d, st, cond_args(ctx, ctx->d_pf_m, r, j, 2));
         GemmArgs a{};
         a.n_dev = n_dev;
@@ -1299,9 +1314,9 @@ static int prefill_batched(tlf_ctx* ctx, int n_seqs, const int* slot_of, const i
         a.row_slot = ctx->d_pf_row_slot + (size_t)r * C;
         a.row_cslot = ctx->d_pf_row_cslot + (size_t)r * C;
         a.row_pos = ctx->d_pf_row_pos + (size_t)r * C;
-        gemm_pf(ctx, ctx->wqkv[j], &ctx->pf_map_X, a, T, st);
-        // attention blocks of loop r: sum over sequences of ceil(count / qblock) <= T / qblock + S
-        launch_pf_attn(md, P, sp, r, j, ctx->d_pf_Q, ctx->d_pf_O, T / P.qblock + S + 1, st,
+        gemm_pf(ctx, ctx->wqkv[j], &ctx->pf_map_X, a, nr, st);
+        // attention blocks of loop r: sum over sequences of ceil(count / qblock) <= nr / qblock + S
+        launch_pf_attn(md, P, sp, r, j, ctx->d_pf_Q, ctx->d_pf_O, nr / P.qblock + S + 1, st,
                        ctx->has_pool_map && ctx->pf_ws ? &ctx->map_pool : nullptr);
         a = GemmArgs{};
         a.n_dev = n_dev;
@@ -1310,15 +1325,15 @@ static int prefill_batched(tlf_ctx* ctx, int n_seqs, const int* slot_of, const i
         a.ldr = md.d;
         a.idx = idx_r;
         a.alpha = cond_args(ctx, ctx->d_pf_m, r, j, 0);
-        gemm_pf(ctx, ctx->wo[j], &ctx->pf_map_O, a, T, st);
-        launch_norm_rows(md.dtype, ctx->d_pf_H, md.d, idx_r, n_dev, 0, T, ctx->d_mlp_norm + (size_t)j * md.d, md.d,
+        gemm_pf(ctx, ctx->wo[j], &ctx->pf_map_O, a, nr, st);
+        launch_norm_rows(md.dtype, ctx->d_pf_H, md.d, idx_r, n_dev, 0, nr, ctx->d_mlp_norm + (size_t)j * md.d, md.d,
                          md.eps, ctx->d_pf_X, md.d, st, cond_args(ctx, ctx->d_pf_m, r, j, 3));
         a = GemmArgs{};
         a.n_dev = n_dev;
         a.epi = EPI_CL_SWIGLU;
         a.md = md;
         a.U = ctx->d_pf_U;
-        gemm_pf(ctx, ctx->wgu[j], &ctx->pf_map_X, a, T, st);
+        gemm_pf(ctx, ctx->wgu[j], &ctx->pf_map_X, a, nr, st);
         a = GemmArgs{};
         a.n_dev = n_dev;
         a.epi = EPI_CL_RESID;
@@ -1326,7 +1341,7 @@ static int prefill_batched(tlf_ctx* ctx, int n_seqs, const int* slot_of, const i
         a.ldr = md.d;
         a.idx = idx_r;
         a.alpha = cond_args(ctx, ctx->d_pf_m, r, j, 1);
-        gemm_pf(ctx, ctx->wd[j], &ctx->pf_map_U, a, T, st);
+        gemm_pf(ctx, ctx->wd[j], &ctx->pf_map_U, a, nr, st);
       }
     }
     if (last_logits && nend > 0) {
