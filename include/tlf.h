@@ -222,6 +222,10 @@ const char* tlf_last_error(const tlf_ctx* ctx);
  *   last_logits  host or device float32 [n_seqs][V] or NULL: logits after
  *                each prompt's last token
  *   loops        host int32 [offsets[n_seqs]] or NULL: loop count per token
+ * The prompts run in chunks of at most prefill_chunk tokens; the call
+ * synchronises `stream` within every chunk (the rows of each loop of a chunk
+ * of more than 256 tokens come to the host to size that loop's launches, and
+ * the loop counts at its end) and before returning.
  * Errors: INVALID_ARG, DUPLICATE_SEQ, CAPACITY, SEQ_TOO_LONG, OUT_OF_PAGES,
  * CUDA, DEVICE. */
 int tlf_prefill(tlf_ctx* ctx, int32_t n_seqs, const uint64_t* seq_ids, const int32_t* offsets,
